@@ -1,0 +1,417 @@
+#!/usr/bin/env python
+"""Throughput of the cache-aware routing + expert-residency step on GB300.
+
+Metric: stream-token-layer route+cache decisions per second.  One step is
+one full pass of the path (router heads, Top-K, refinement, access,
+retention, accounting) over the whole workload: every stream, token and
+layer, from a cold cache state.  Inputs are synthetic (seeded AR(1) hidden
+states and N(0, 1/d) router weights) with the shapes of the named backbone
+and already resident in HBM when the timed region starts; the hidden states
+(12.9 GB for the Qwen3-30B shape) are far larger than L2, so no flush is
+needed between steps.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Multi-GPU (torchrun): streams are independent, every rank runs its own
+streams (weak scaling), no data-path collective; timing is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import crc_synth as S  # noqa: E402
+
+METRIC = "stream-token-layer route+cache decisions/sec"
+UNIT = "decisions/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=S.QWEN3_30B.name, choices=sorted(S.WORKLOADS))
+    ap.add_argument("--chunk", type=int, default=0, help="tokens per workspace chunk (0 = auto)")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------------------- #
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def algorithmic(w, units: int, heads: int):
+    """Algorithmic flops and HBM bytes of the fused step for `units` decisions:
+    2*d*H*N flops per unit; bf16 hidden state read once (2d bytes), the
+    weights once per pass, trace-free accounting."""
+    flops = 2.0 * w.d * heads * w.N * units
+    bytes_ = 2.0 * w.d * units + 2.0 * w.L * heads * w.N * w.d
+    return flops, bytes_
+
+
+def workload_config(w, chunk=None):
+    cfg = {"workload": f"{w.name}: L={w.L} N={w.N} K={w.K} d={w.d} C={w.C} R={w.R} "
+                       f"B={w.B} T={w.T}",
+           "L": w.L, "N": w.N, "K": w.K, "d": w.d, "C": w.C, "R": w.R,
+           "streams": w.B, "tokens": w.T, "expert_bytes": w.expert_bytes,
+           "rho_t": w.rho_t, "rho_l": w.rho_l,
+           "l2": "inputs larger than L2 (hidden states %.1f GB per step), no flush"
+                 % (2.0 * w.units * w.d / 1e9)}
+    if chunk:
+        cfg["chunk_tokens"] = chunk
+    return cfg
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.t.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [x.strip() for x in ln.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_id_for_smi(torch, dev: int) -> str:
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        if vis:
+            return vis.split(",")[dev]
+        return str(dev)
+
+
+def source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_04895_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(kernel: str, workload: str):
+    """DRAM bytes per unit from a committed ncu capture, if taken on the current sources."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+    except (OSError, ValueError):
+        return None, None
+    e = d.get(kernel, {}).get(workload)
+    if not e or e.get("src_sha") != source_hash():
+        return None, None
+    return e.get("dram_bytes_per_unit"), e.get("source")
+
+
+# --------------------------------------------------------------------------- #
+def cpu_oracle_sample(w, seconds: float):
+    """Times the CPU oracle (as it stands) on a bounded sample of workload w:
+    the first streams and tokens, all layers, fp64 router heads + scan."""
+    import numpy as np
+
+    import oracle
+    oracle.build()
+    threads = oracle.default_threads()
+    Wb = S.weights(w, seed=0)
+
+    def run(nb, nt):
+        h = S.hidden(w.with_(B=nb), seed=0, T=nt)
+        t0 = time.perf_counter()
+        res = oracle.run(h, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
+        dt = time.perf_counter() - t0
+        return dt, res
+
+    pilot_t = min(8, w.T)
+    dt, _ = run(1, pilot_t)
+    rate = (pilot_t * w.L) / max(dt, 1e-6)
+    want_units = rate * seconds
+    nt = int(min(w.T, max(pilot_t, want_units // w.L)))
+    nb = int(min(w.B, max(1, want_units // (w.L * nt))))
+    dt, res = run(nb, nt)
+    units = nb * nt * w.L
+    del res, np
+    return {"value": units / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{nb} stream(s) x {nt} tokens x {w.L} layers = {units} decisions "
+                      f"(fp64 router heads + literal scan), {dt:.1f} s wall"}, units, dt
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = S.WORKLOADS[args.workload]
+    import oracle
+    oracle.build()
+    threads = oracle.default_threads()
+    Wb = S.weights(w, seed=0)
+    # size one step at a few seconds of oracle time
+    h1 = S.hidden(w.with_(B=1), seed=0, T=min(4, w.T))
+    t0 = time.perf_counter()
+    oracle.run(h1, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
+    rate = h1.shape[1] * w.L / max(time.perf_counter() - t0, 1e-6)
+    budget = max(1.0, min(6.0, 150.0 / max(1, args.steps + args.warmup)))
+    nt = int(min(w.T, max(4, rate * budget // w.L)))
+    h = S.hidden(w.with_(B=1), seed=0, T=nt)
+    for _ in range(args.warmup):
+        oracle.run(h, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.run(h, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
+    dt = time.perf_counter() - t0
+    units = nt * w.L
+    value = units * args.steps / dt
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(w), "impl": "reference",
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"1 stream x {nt} tokens x {w.L} layers = {units} decisions "
+                                   f"per step (fp64 router heads + literal scan)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# --------------------------------------------------------------------------- #
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    from paper_2609_04895_gb300 import build as B_
+    B_.build()
+    import paper_2609_04895_gb300 as P
+    C = P.crc
+
+    w = S.WORKLOADS[args.workload]
+    p = P.problem_of(w)
+    heads = 3 if w.R > 0 else 2
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+
+    # inputs, resident in HBM before timing (untimed generation)
+    Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
+    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
+                           rho_l=w.rho_l, device=dev)
+    chunk = args.chunk or w.T
+    ws = torch.empty(C.crc_workspace_bytes(p, chunk), dtype=torch.uint8, device=dev)
+    st = P.State(p, device=dev)
+    torch.cuda.synchronize()
+
+    def step():
+        st.init()
+        C.crc_route_and_cache(p, hd.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes, None,
+                              ws.data_ptr(), ws.numel(), stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    stats = st.read()
+    assert stats["error"] == 0 and stats["tokens"] == w.T, stats
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(gpu_id_for_smi(torch, local)) as clk:
+        C.crc_profile_begin()
+        n0 = C.crc_launch_count()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        launches = C.crc_launch_count() - n0
+        kt = C.crc_profile_end()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+    ms_per_step = ms / args.steps
+    units_all = w.units * world
+    value = units_all / (ms_per_step / 1000.0)
+
+    # roofline of the dominant kernel, timed live over the timed region
+    pk, pk_src = peaks()
+    dom = max(("router", "scan"), key=lambda k: kt[k]["ms"])
+    avg_ms = kt[dom]["ms"] / max(1, kt[dom]["launches"])
+    if dom == "router":
+        flops = 2.0 * w.d * heads * w.N * w.units * args.steps
+        bytes_ = (2.0 * w.d + 4.0 * heads * w.N) * w.units * args.steps
+        t_s = kt[dom]["ms"] / 1000.0
+        f_frac = flops / t_s / (pk["bf16_tflops"] * 1e12)
+        b_frac = bytes_ / t_s / (pk["hbm_gbs"] * 1e9)
+        if flops / (pk["bf16_tflops"] * 1e12) >= bytes_ / (pk["hbm_gbs"] * 1e9):
+            roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": pk["bf16_tflops"],
+                    "unit": "TFLOP/s", "frac": f_frac}
+        else:
+            roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
+                    "unit": "GB/s", "frac": b_frac}
+        kname = f"router_heads_kernel<{w.N},{heads}>"
+    else:
+        bytes_ = 4.0 * heads * w.N * w.units * args.steps
+        t_s = kt[dom]["ms"] / 1000.0
+        roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "frac": bytes_ / t_s / (pk["hbm_gbs"] * 1e9)}
+        kname = "cache_scan_kernel"
+    per_unit, src = committed_traffic(kname, w.name)
+    units_per_launch = w.units * args.steps / max(1, kt[dom]["launches"])
+    roof["traffic"] = None if per_unit is None else per_unit * units_per_launch
+    roof.update({"kernel": kname, "peak_source": f"{pk_src} ({'burst' if roof['bound'] == 'tensor' else 'copy'})",
+                 "avg_launch_ms": avg_ms, "launches": kt[dom]["launches"],
+                 "share_of_step": kt[dom]["ms"] / ms if ms else None})
+    # whole-path roofline (spec definition): max(flops at bf16 peak, bytes at HBM)
+    fl, by = algorithmic(w, w.units, heads)
+    t_roof = max(fl / (pk["bf16_tflops"] * 1e12), by / (pk["hbm_gbs"] * 1e9))
+    path_roof = {"t_roof_ms": 1000 * t_roof, "frac": 1000 * t_roof / ms_per_step,
+                 "bound": "tensor" if fl / (pk["bf16_tflops"] * 1e12) >= by / (pk["hbm_gbs"] * 1e9)
+                 else "hbm"}
+    kernels = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / args.steps}
+               for k, v in kt.items() if v["launches"]}
+
+    # end to end through the C ABI from pinned host memory
+    e2e = None
+    if not args.no_e2e:
+        h_host = torch.empty(hd.shape, dtype=hd.dtype, pin_memory=True)
+        h_host.copy_(hd)
+        del hd
+        torch.cuda.empty_cache()
+        h_dev = torch.empty(h_host.shape, dtype=h_host.dtype, device=dev)
+        torch.cuda.synchronize()
+
+        def e2e_step():
+            h_dev.copy_(h_host, non_blocking=True)
+            st.init()
+            C.crc_route_and_cache(p, h_dev.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes,
+                                  None, ws.data_ptr(), ws.numel(), stream)
+            return st.read()      # synchronises; reads the step's counters back
+
+        for _ in range(2):
+            e2e_step()
+        if world > 1:
+            dist.barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            r = e2e_step()
+        dt = time.perf_counter() - t0
+        if world > 1:
+            t = torch.tensor([dt], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            dt = float(t.item())
+        assert r["error"] == 0
+        e2e = {"value": units_all * args.steps / dt, "unit": UNIT,
+               "h2d_bytes_per_step": int(h_host.numel() * h_host.element_size()),
+               "d2h_bytes_per_step": int(256 + p.B * p.L * 64),
+               "ms_per_step": 1000 * dt / args.steps}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu, _, _ = cpu_oracle_sample(w, args.cpu_seconds)
+
+    if rank == 0:
+        m = P.metrics(stats, p)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "config": workload_config(w, chunk),
+            "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
+            "clocks": clk.summary(),
+            "policy": {"hit": m["hit"], "adj_hit": m["adj_hit"],
+                       "load_MB_per_token": m["load_per_token_bytes"] / 1e6},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

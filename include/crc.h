@@ -1,0 +1,213 @@
+/*
+ * crc.h -- C ABI of the GB300 (sm_103a) cache-aware MoE routing library.
+ *
+ * For a batch of B independent decode streams, T tokens and L MoE layers
+ * with N routed experts each, the library computes the per-token, per-layer
+ * routing and expert-residency step of cache-aware MoE decoding ("Cache-Aware
+ * Joint Router Adaptation for Memory-Efficient MoE Inference"):
+ *
+ *   p^R = softmax(W^R_l h), S = TopK(p^R)               (Sec. 2)
+ *   p^T = softmax(W^T_l h), s^T = p^R + p^T             (Sec. 3.2)
+ *   p^S = softmax(W^S_l h), s^ST = s^T_{t-1} + p^S_rho  (Sec. 3.3)
+ *   pre-access refinement (Algorithm 2, R > 0), access, post-access
+ *   retention UpdateCache (Algorithm 1) on a C-slot cache per (stream, layer),
+ *   counting accesses, demand misses and proactive loads (Sec. 4.1 Metrics).
+ *
+ * Notation: the paper's cache capacity B is called C here; B here is the
+ * number of independent decode streams.  Layers and tokens are 0-indexed,
+ * so the causal predecessor is rho(t,0) = (t-1, L-1), rho(t,l) = (t, l-1).
+ *
+ * Conventions for every entry point:
+ *  - Pointers named *_dev are device pointers the caller allocated (the
+ *    library allocates no device memory except where stated); *_host are
+ *    host pointers.  bf16 data is passed as uint16_t bit patterns.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls are
+ *    asynchronous on it unless stated; they return after enqueueing.
+ *  - Return value: CRC_OK (0) or an error code below.  Argument errors are
+ *    detected on the host before anything is enqueued.  Errors found on the
+ *    device (a bounded wait that ran out, a state mismatch) are latched in
+ *    the state's error word and reported by crc_state_read(), or, for calls
+ *    without a state, by crc_device_error().  Nothing aborts or prints.
+ *  - Policy decisions use one total order: score descending, then expert
+ *    index ascending.  Top-K / Top-R take its first elements; every argmin
+ *    takes its last (smallest score, ties to the highest index).  The
+ *    refinement test is strict.  No refinement at a stream's first token.
+ *    Caches start empty.  Scores are probabilities (finite, >= 0).
+ *  - Limits: 16 <= N <= 128 with N % 16 == 0 for the router entry points
+ *    (N <= 256 for crc_cache_scan); 1 <= K <= min(C, 32); K <= C <= N;
+ *    0 <= R <= N; d % 8 == 0; L >= 1; B >= 1.
+ */
+#ifndef CRC_H
+#define CRC_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    CRC_OK = 0,
+    CRC_EINVAL = 1,        /* null / misaligned pointer, bad size, T < 0      */
+    CRC_EUNSUPPORTED = 2,  /* sizes outside the limits above                  */
+    CRC_ECUDA = 3,         /* a CUDA runtime call or launch failed            */
+    CRC_ETIMEOUT = 4,      /* a bounded device wait ran out (latched)         */
+    CRC_ESTATE = 5,        /* state buffer too small, uninitialised or made
+                              for another problem (latched when seen on GPU)  */
+    CRC_EDEVICE = 6        /* other device-side failure (latched)             */
+};
+
+/* The problem statement (Sec. 2): sizes and budgets.  One per state. */
+typedef struct crc_problem {
+    int32_t L;              /* MoE layers                                     */
+    int32_t N;              /* routed experts per layer                       */
+    int32_t K;              /* native Top-K                                   */
+    int32_t d;              /* hidden size                                    */
+    int32_t C;              /* cache slots per layer (the paper's B)          */
+    int32_t R;              /* refinement budget; 0 = update-only mode        */
+    int32_t B;              /* independent decode streams                     */
+    int32_t reserved;       /* must be 0                                      */
+    uint64_t expert_bytes;  /* bytes of one expert transfer (S_exp)           */
+} crc_problem;
+
+/* Optional per-access trace of one call, device pointers, each may be NULL.
+ * T is the call's token count and t the token index within the call. */
+typedef struct crc_trace {
+    uint8_t *topk_dev;       /* [B][T][L][K] native Top-K, rank order          */
+    uint8_t *misses_dev;     /* [B][T][L] demand misses |S \ C~|               */
+    uint8_t *proactive_dev;  /* [B][T][L] proactive loads of the refinement    */
+} crc_trace;
+
+/* Totals over all streams and layers since crc_state_init (Sec. 4.1). */
+typedef struct crc_stats {
+    uint64_t accesses;       /* A = L * K * tokens * B                         */
+    uint64_t hits;           /* A - D                                          */
+    uint64_t misses;         /* D, demand misses                               */
+    uint64_t proactive;      /* P, proactive loads                             */
+    uint64_t traffic_bytes;  /* (D + P) * expert_bytes                         */
+    uint64_t tokens;         /* tokens processed per stream                    */
+    uint32_t error;          /* latched device error code, CRC_OK if none      */
+    uint32_t reserved;
+} crc_stats;
+
+/* ------------------------------------------------------------------------ */
+/* State: a caller-owned device buffer holding, per (stream, layer), the    */
+/* cache set C_{t,l} (bitmask), the carried retention score s^T_{t-1,l}     */
+/* (= a^T_{t,l}, fp32 [N]) and hit / miss / proactive counters; per stream  */
+/* the carried Spatio prediction p^S_{t-1,L-1} (the wrap-around             */
+/* predecessor of layer 0); and the next token index.  Successive calls on  */
+/* one state continue the same streams: processing T tokens in chunks gives */
+/* bit-identical results to one call.  Two calls on one state must not run  */
+/* concurrently.                                                            */
+/* ------------------------------------------------------------------------ */
+
+/* Bytes needed for the state of problem p (0 if p is invalid). */
+size_t crc_state_bytes(const crc_problem *p);
+
+/* Cold start: empty caches, zero counters, token 0.  state_dev must be
+ * 256-byte aligned and hold crc_state_bytes(p) bytes.  Asynchronous. */
+int crc_state_init(const crc_problem *p, void *state_dev, size_t state_bytes, void *stream);
+
+/* Synchronises `stream`, then reads the state back: totals into *out
+ * (required); optionally cache bitmasks [B][L][ceil(N/32)] (bit e % 32 of
+ * word e / 32 set when expert e is resident), the carried retention scores
+ * [B][L][N] and per-(stream, layer) counters [B][L][3] = hits, misses,
+ * proactive.  Returns the latched device error if there is one. */
+int crc_state_read(const crc_problem *p, const void *state_dev, size_t state_bytes,
+                   crc_stats *out, uint32_t *cache_bits_host, float *retention_host,
+                   uint64_t *chain_counters_host, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Hot path                                                                 */
+/* ------------------------------------------------------------------------ */
+
+/* Router heads (Sec. 2, 3.2, 3.3): for every unit (b, t, l),
+ *   scores[b][t][l][x][:] = softmax(W_cat[l][x*N:(x+1)*N] . hidden[b][t][l]),
+ * x = 0 (native R), 1 (Temporal T), 2 (Spatio S); heads = 2 skips S (the
+ * S slot of `scores` is then left untouched).  One bf16 GEMM per layer on
+ * the tensor cores with fp32 accumulation, softmax in fp32.
+ *   hidden_dev  bf16 [B][T][L][d], 16-byte aligned
+ *   w_cat_dev   bf16 [L][3N][d], heads ordered R, T, S, 16-byte aligned
+ *   scores_dev  fp32 [B][T][L][3][N], 16-byte aligned
+ * T = 0 is a no-op.  Device-side failures: crc_device_error(). */
+int crc_route_scores(const crc_problem *p, const uint16_t *hidden_dev,
+                     const uint16_t *w_cat_dev, int32_t T, int32_t heads,
+                     float *scores_dev, void *stream);
+
+/* Cache simulation over T tokens (Algorithm 2 with Algorithm 1, Sec. 4.1
+ * accounting) from router probabilities, one warp per (stream, layer):
+ *   scores_dev  fp32 [B][T][L][3][N] as written by crc_route_scores (the S
+ *               head is read only when R > 0), 16-byte aligned.
+ * Continues the streams held in `state_dev`; `trace` may be NULL. */
+int crc_cache_scan(const crc_problem *p, const float *scores_dev, int32_t T,
+                   void *state_dev, size_t state_bytes, const crc_trace *trace,
+                   void *stream);
+
+/* Bytes of workspace crc_route_and_cache uses to process `chunk_tokens`
+ * tokens per pass (the router scores of one chunk). */
+size_t crc_workspace_bytes(const crc_problem *p, int32_t chunk_tokens);
+
+/* The whole step: router heads and cache simulation over T tokens, the
+ * same results as crc_route_scores followed by crc_cache_scan (bit for bit).
+ * hidden_dev bf16 [B][T][L][d]; w_cat_dev bf16 [L][3N][d] (the S head is
+ * not computed when R = 0).  The router scores never leave the workspace:
+ * workspace_dev holds the scores of one chunk of tokens; the chunk length is
+ * the largest that fits in workspace_bytes (at least one token must fit, see
+ * crc_workspace_bytes).  256-byte alignment for the workspace. */
+int crc_route_and_cache(const crc_problem *p, const uint16_t *hidden_dev,
+                        const uint16_t *w_cat_dev, int32_t T, void *state_dev,
+                        size_t state_bytes, const crc_trace *trace,
+                        void *workspace_dev, size_t workspace_bytes, void *stream);
+
+/* ------------------------------------------------------------------------ */
+/* Support                                                                  */
+/* ------------------------------------------------------------------------ */
+
+/* Synchronises the device and returns (then clears) the error latched by
+ * calls without a state (crc_route_scores), CRC_OK if none. */
+int crc_device_error(void);
+
+/* Number of kernels the library has launched in this process. */
+uint64_t crc_launch_count(void);
+
+/* Optional per-kernel timing.  Between crc_profile_begin() and
+ * crc_profile_end(), every kernel the library launches is bracketed by two
+ * CUDA events recorded on its launching stream.  crc_profile_end()
+ * synchronises those events and returns, per kernel kind, the number of
+ * launches and their summed device time in milliseconds.  Host-side
+ * bookkeeping only; off by default.  Not thread-safe against concurrent
+ * library calls from other host threads. */
+enum { CRC_KERNEL_ROUTER = 0, CRC_KERNEL_SCAN = 1, CRC_KERNEL_STATE = 2, CRC_KERNEL_SYNTH = 3,
+       CRC_KERNEL_KINDS = 8 };
+typedef struct crc_kernel_times {
+    uint64_t launches[CRC_KERNEL_KINDS];
+    double ms[CRC_KERNEL_KINDS];
+} crc_kernel_times;
+int crc_profile_begin(void);
+int crc_profile_end(crc_kernel_times *out);
+
+/* Message for an error code (static string). */
+const char *crc_strerror(int code);
+
+/* Seeded synthetic inputs (not part of the method).  Same definition as the
+ * host generator: Philox4x32-10 counters, Irwin-Hall(4) unit normals,
+ * separable AR(1) over layers then tokens, bf16 round-to-nearest-even.
+ * crc_synth_hidden writes tokens [t0, t0 + T) of hidden bf16 [B][T][L][d]
+ * (the chunk); carry_dev fp32 [B][L][d] holds h of token t0 - 1 on entry
+ * (ignored when t0 == 0) and of token t0 + T - 1 on exit.  attempts_dev
+ * (uint8 [B][T][L], may be NULL) selects re-drawn innovations per unit.
+ * crc_synth_weights writes W_cat bf16 [L][3N][d] ~ N(0, 1/d); copy_init
+ * copies native rows into the other heads (W^T_l = W^R_l,
+ * W^S_l = W^R_{(l+1) mod L}). */
+int crc_synth_hidden(int32_t B, int32_t T, int32_t L, int32_t d, int32_t t0,
+                     uint32_t seed, double rho_t, double rho_l,
+                     const uint8_t *attempts_dev, uint16_t *hidden_dev,
+                     float *carry_dev, void *stream);
+int crc_synth_weights(int32_t L, int32_t N, int32_t d, uint32_t seed, int32_t copy_init,
+                      uint16_t *w_cat_dev, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CRC_H */

@@ -1,0 +1,322 @@
+"""ctypes binding of the CUDA library (include/crc.h), names as in the C ABI.
+
+Argument marshalling only: every step of the routing and cache path runs in
+the library's kernels.  PyTorch supplies device memory and streams.  There
+is no fallback: if libcrc.so is missing or a call fails, an exception is
+raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libcrc.so")
+
+CRC_OK, CRC_EINVAL, CRC_EUNSUPPORTED, CRC_ECUDA, CRC_ETIMEOUT, CRC_ESTATE, CRC_EDEVICE = range(7)
+
+
+class crc_problem(ctypes.Structure):
+    _fields_ = [("L", ctypes.c_int32), ("N", ctypes.c_int32), ("K", ctypes.c_int32),
+                ("d", ctypes.c_int32), ("C", ctypes.c_int32), ("R", ctypes.c_int32),
+                ("B", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("expert_bytes", ctypes.c_uint64)]
+
+
+class crc_trace(ctypes.Structure):
+    _fields_ = [("topk_dev", ctypes.c_void_p), ("misses_dev", ctypes.c_void_p),
+                ("proactive_dev", ctypes.c_void_p)]
+
+
+class crc_stats(ctypes.Structure):
+    _fields_ = [("accesses", ctypes.c_uint64), ("hits", ctypes.c_uint64),
+                ("misses", ctypes.c_uint64), ("proactive", ctypes.c_uint64),
+                ("traffic_bytes", ctypes.c_uint64), ("tokens", ctypes.c_uint64),
+                ("error", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
+
+
+KERNEL_KINDS = {"router": 0, "scan": 1, "state": 2, "synth": 3}
+
+
+class crc_kernel_times(ctypes.Structure):
+    _fields_ = [("launches", ctypes.c_uint64 * 8), ("ms", ctypes.c_double * 8)]
+
+
+class CrcError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        self.code = code
+        super().__init__(f"{what}: {crc_strerror(code)} (code {code})")
+
+
+_lib = None
+_lock = threading.Lock()
+
+# (name, restype, argtypes) of every exported symbol
+P, I32, U32, U64, SZ, D = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint32, ctypes.c_uint64,
+                           ctypes.c_size_t, ctypes.c_double)
+PP = ctypes.POINTER(crc_problem)
+EXPORTS = [
+    ("crc_state_bytes", SZ, [PP]),
+    ("crc_state_init", ctypes.c_int, [PP, P, SZ, P]),
+    ("crc_state_read", ctypes.c_int, [PP, P, SZ, ctypes.POINTER(crc_stats), P, P, P, P]),
+    ("crc_route_scores", ctypes.c_int, [PP, P, P, I32, I32, P, P]),
+    ("crc_cache_scan", ctypes.c_int, [PP, P, I32, P, SZ, ctypes.POINTER(crc_trace), P]),
+    ("crc_workspace_bytes", SZ, [PP, I32]),
+    ("crc_route_and_cache", ctypes.c_int,
+     [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P, SZ, P]),
+    ("crc_device_error", ctypes.c_int, []),
+    ("crc_launch_count", U64, []),
+    ("crc_strerror", ctypes.c_char_p, [ctypes.c_int]),
+    ("crc_profile_begin", ctypes.c_int, []),
+    ("crc_profile_end", ctypes.c_int, [ctypes.POINTER(crc_kernel_times)]),
+    ("crc_synth_hidden", ctypes.c_int, [I32, I32, I32, I32, I32, U32, D, D, P, P, P, P]),
+    ("crc_synth_weights", ctypes.c_int, [I32, I32, I32, U32, I32, P, P]),
+]
+
+
+def load(path: str = LIB_PATH):
+    """Load libcrc.so (built by paper_2609_04895_gb300.build); raises if absent."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(path):
+                raise ImportError(
+                    f"CUDA library not built: {path} (run paper_2609_04895_gb300.build.build())")
+            lib = ctypes.CDLL(path)
+            for name, res, args in EXPORTS:
+                f = getattr(lib, name)
+                f.restype = res
+                f.argtypes = args
+            _lib = lib
+    return _lib
+
+
+def _ck(rc: int, what: str):
+    if rc != CRC_OK:
+        raise CrcError(rc, what)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ptr(t) -> int:
+    if t is None:
+        return None
+    return t.data_ptr()
+
+
+# --------------------------------------------------------------------------- #
+# C-ABI names
+# --------------------------------------------------------------------------- #
+def crc_strerror(code: int) -> str:
+    try:
+        return load().crc_strerror(code).decode()
+    except ImportError:
+        return f"error {code}"
+
+
+def crc_state_bytes(p: crc_problem) -> int:
+    return int(load().crc_state_bytes(ctypes.byref(p)))
+
+
+def crc_state_init(p: crc_problem, state_ptr: int, state_bytes: int, stream=None):
+    _ck(load().crc_state_init(ctypes.byref(p), state_ptr, state_bytes, _stream(stream)),
+        "crc_state_init")
+
+
+def crc_state_read(p: crc_problem, state_ptr: int, state_bytes: int, stream=None,
+                   want_caches: bool = False, want_retention: bool = False,
+                   want_chain_counters: bool = False) -> dict:
+    st = crc_stats()
+    B, L, N = p.B, p.L, p.N
+    bits = np.zeros((B, L, (N + 31) // 32), np.uint32) if want_caches else None
+    ret = np.zeros((B, L, N), np.float32) if want_retention else None
+    cc = np.zeros((B, L, 3), np.uint64) if want_chain_counters else None
+    rc = load().crc_state_read(ctypes.byref(p), state_ptr, state_bytes, ctypes.byref(st),
+                               None if bits is None else bits.ctypes.data,
+                               None if ret is None else ret.ctypes.data,
+                               None if cc is None else cc.ctypes.data, _stream(stream))
+    _ck(rc, "crc_state_read")
+    out = {f: int(getattr(st, f)) for f, _ in crc_stats._fields_ if f != "reserved"}
+    out.update(cache_bits=bits, retention=ret, chain_counters=cc)
+    return out
+
+
+def crc_route_scores(p: crc_problem, hidden_ptr: int, w_ptr: int, T: int, heads: int,
+                     scores_ptr: int, stream=None):
+    _ck(load().crc_route_scores(ctypes.byref(p), hidden_ptr, w_ptr, T, heads, scores_ptr,
+                                _stream(stream)), "crc_route_scores")
+
+
+def crc_cache_scan(p: crc_problem, scores_ptr: int, T: int, state_ptr: int, state_bytes: int,
+                   trace: crc_trace | None = None, stream=None):
+    _ck(load().crc_cache_scan(ctypes.byref(p), scores_ptr, T, state_ptr, state_bytes,
+                              None if trace is None else ctypes.byref(trace), _stream(stream)),
+        "crc_cache_scan")
+
+
+def crc_workspace_bytes(p: crc_problem, chunk_tokens: int) -> int:
+    return int(load().crc_workspace_bytes(ctypes.byref(p), chunk_tokens))
+
+
+def crc_route_and_cache(p: crc_problem, hidden_ptr: int, w_ptr: int, T: int, state_ptr: int,
+                        state_bytes: int, trace: crc_trace | None, ws_ptr: int, ws_bytes: int,
+                        stream=None):
+    _ck(load().crc_route_and_cache(ctypes.byref(p), hidden_ptr, w_ptr, T, state_ptr, state_bytes,
+                                   None if trace is None else ctypes.byref(trace), ws_ptr,
+                                   ws_bytes, _stream(stream)), "crc_route_and_cache")
+
+
+def crc_device_error() -> int:
+    return int(load().crc_device_error())
+
+
+def crc_launch_count() -> int:
+    return int(load().crc_launch_count())
+
+
+def crc_profile_begin():
+    _ck(load().crc_profile_begin(), "crc_profile_begin")
+
+
+def crc_profile_end() -> dict:
+    kt = crc_kernel_times()
+    _ck(load().crc_profile_end(ctypes.byref(kt)), "crc_profile_end")
+    return {k: {"launches": int(kt.launches[i]), "ms": float(kt.ms[i])}
+            for k, i in KERNEL_KINDS.items()}
+
+
+def crc_synth_hidden(B, T, L, d, t0, seed, rho_t, rho_l, attempts_ptr, hidden_ptr, carry_ptr,
+                     stream=None):
+    _ck(load().crc_synth_hidden(B, T, L, d, t0, seed, rho_t, rho_l, attempts_ptr, hidden_ptr,
+                                carry_ptr, _stream(stream)), "crc_synth_hidden")
+
+
+def crc_synth_weights(L, N, d, seed, copy_init, w_ptr, stream=None):
+    _ck(load().crc_synth_weights(L, N, d, seed, int(copy_init), w_ptr, _stream(stream)),
+        "crc_synth_weights")
+
+
+# --------------------------------------------------------------------------- #
+# torch conveniences (allocation and marshalling only)
+# --------------------------------------------------------------------------- #
+def problem(L, N, K, d, C, R, B, expert_bytes) -> crc_problem:
+    return crc_problem(L=L, N=N, K=K, d=d, C=C, R=R, B=B, reserved=0,
+                       expert_bytes=int(expert_bytes))
+
+
+def problem_of(w) -> crc_problem:
+    """crc_problem from an object with fields L, N, K, d, C, R, B, expert_bytes."""
+    return problem(w.L, w.N, w.K, w.d, w.C, w.R, w.B, w.expert_bytes)
+
+
+class State:
+    """A cache state in device memory (torch-allocated, 256-byte aligned)."""
+
+    def __init__(self, p: crc_problem, device="cuda", stream=None):
+        import torch
+        self.p = p
+        self.nbytes = crc_state_bytes(p)
+        if self.nbytes == 0:
+            raise CrcError(CRC_EINVAL, "crc_state_bytes")
+        self.buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device)
+        assert self.buf.data_ptr() % 256 == 0
+        self.init(stream)
+
+    @property
+    def ptr(self) -> int:
+        return self.buf.data_ptr()
+
+    def init(self, stream=None):
+        crc_state_init(self.p, self.ptr, self.nbytes, stream)
+
+    def read(self, stream=None, **kw) -> dict:
+        return crc_state_read(self.p, self.ptr, self.nbytes, stream, **kw)
+
+
+@dataclass
+class Trace:
+    topk: object
+    misses: object
+    proactive: object
+
+    @staticmethod
+    def alloc(p: crc_problem, T: int, device="cuda") -> "Trace":
+        import torch
+        return Trace(torch.zeros((p.B, T, p.L, p.K), dtype=torch.uint8, device=device),
+                     torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device),
+                     torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device))
+
+    def c(self) -> crc_trace:
+        return crc_trace(_ptr(self.topk), _ptr(self.misses), _ptr(self.proactive))
+
+
+def route_scores(p: crc_problem, hidden, w_cat, heads: int = 3, out=None, stream=None):
+    import torch
+    B, T, L, d = hidden.shape
+    if out is None:
+        out = torch.empty((B, T, L, 3, p.N), dtype=torch.float32, device=hidden.device)
+    crc_route_scores(p, hidden.data_ptr(), w_cat.data_ptr(), T, heads, out.data_ptr(), stream)
+    return out
+
+
+def cache_scan(p: crc_problem, scores, state: State, trace: Trace | None = None, stream=None):
+    T = scores.shape[1]
+    crc_cache_scan(p, scores.data_ptr(), T, state.ptr, state.nbytes,
+                   None if trace is None else trace.c(), stream)
+
+
+def route_and_cache(p: crc_problem, hidden, w_cat, state: State, trace: Trace | None = None,
+                    workspace=None, stream=None):
+    import torch
+    T = hidden.shape[1]
+    if workspace is None:
+        workspace = torch.empty(crc_workspace_bytes(p, T), dtype=torch.uint8,
+                                device=hidden.device)
+    crc_route_and_cache(p, hidden.data_ptr(), w_cat.data_ptr(), T, state.ptr, state.nbytes,
+                        None if trace is None else trace.c(), workspace.data_ptr(),
+                        workspace.numel() * workspace.element_size(), stream)
+    return workspace
+
+
+def synth_weights(L, N, d, seed=0, copy_init=False, device="cuda", stream=None):
+    import torch
+    w = torch.empty((L, 3 * N, d), dtype=torch.bfloat16, device=device)
+    crc_synth_weights(L, N, d, seed, copy_init, w.data_ptr(), stream)
+    return w
+
+
+def synth_hidden(B, T, L, d, seed=0, rho_t=0.9, rho_l=0.8, t0=0, carry=None, attempts=None,
+                 out=None, device="cuda", stream=None):
+    """Tokens [t0, t0+T) of the synthetic hidden-state field; returns (hidden, carry)."""
+    import torch
+    if out is None:
+        out = torch.empty((B, T, L, d), dtype=torch.bfloat16, device=device)
+    if carry is None:
+        carry = torch.zeros((B, L, d), dtype=torch.float32, device=device)
+    crc_synth_hidden(B, T, L, d, t0, seed, rho_t, rho_l, _ptr(attempts), out.data_ptr(),
+                     carry.data_ptr(), stream)
+    return out, carry
+
+
+def metrics(stats: dict, p: crc_problem) -> dict:
+    """Hit, AdjHit and Load/token (bytes per decode token) of Sec. 4.1 from
+    the totals of crc_state_read; decode tokens = streams x tokens per stream."""
+    A, D, Pn = stats["accesses"], stats["misses"], stats["proactive"]
+    tokens = stats["tokens"] * p.B
+    return {
+        "hit": 1.0 - D / A if A else float("nan"),
+        "adj_hit": (A - D) / (A + Pn) if A + Pn else float("nan"),
+        "traffic_bytes": (D + Pn) * p.expert_bytes,
+        "load_per_token_bytes": (D + Pn) * p.expert_bytes / tokens if tokens else 0.0,
+    }

@@ -1,0 +1,48 @@
+// Host-side internals shared by the translation units of the library.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/crc.h"
+
+namespace crc {
+
+// Count of kernels launched by the library (reported by crc_launch_count).
+void note_launch();
+
+// Brackets one kernel launch with CUDA events on its stream while
+// crc_profile_begin() .. crc_profile_end() is active; otherwise a no-op.
+struct ProfScope {
+    ProfScope(int kind, cudaStream_t stream);
+    ~ProfScope();
+    int slot;
+    cudaStream_t stream;
+};
+
+// Library-wide device error word for calls without a state.
+uint32_t* device_error_word();
+
+// Streaming multiprocessors of the current device.
+int sm_count();
+
+// Router heads over tokens [t_begin, t_begin + T_ext) of hidden [B][T_total][L][d];
+// scores [B][T_ext][L][3][N].
+int launch_router(const crc_problem& p, const uint16_t* hidden, int T_total, int t_begin,
+                  int T_ext, const uint16_t* w_cat, int heads, float* scores,
+                  uint32_t* err_word, cudaStream_t stream);
+
+// Cache scan over T tokens of scores [B][T][L][3][N]; trace arrays are
+// [B][trace_T][L][..] and this call writes tokens trace_t0 .. trace_t0 + T - 1.
+int launch_scan(const crc_problem& p, const float* scores, int T, void* state,
+                const crc_trace* trace, int trace_T, int trace_t0, cudaStream_t stream);
+
+int launch_state_init(const crc_problem& p, void* state, size_t bytes, cudaStream_t stream);
+
+int launch_synth_hidden(int B, int T, int L, int d, int t0, uint32_t seed, double rho_t,
+                        double rho_l, const uint8_t* attempts, uint16_t* out, float* carry,
+                        cudaStream_t stream);
+int launch_synth_weights(int L, int N, int d, uint32_t seed, int copy_init, uint16_t* out,
+                         cudaStream_t stream);
+
+}  // namespace crc

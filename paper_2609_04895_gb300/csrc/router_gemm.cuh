@@ -1,0 +1,285 @@
+// Router heads on the 5th-generation tensor cores (sm_103a).
+//
+// For one layer l the three heads are one GEMM (Sec. 2, 3.2, 3.3):
+//   Z_l[rows, H*N] = H_l[rows, d] . W_cat,l[H*N, d]^T,   rows = (stream, token)
+// bf16 operands staged by TMA into 128-byte-swizzled shared memory, fp32
+// accumulators in TMEM (tcgen05.mma issued by one thread), then a per-row
+// softmax of every head read back with tcgen05.ld.  A tile is 128 rows =
+// SB streams x TB tokens of one layer.  The kernel is persistent: one CTA
+// per SM walks tiles in layer-major order so that the CTAs running together
+// share one layer's weights in L2.
+//
+// Warp roles (192 threads): warp 0 = TMA producer, warp 1 = TMEM allocator
+// and MMA issuer, warps 2..5 = epilogue (warp w reads TMEM lanes
+// 32*(w%4) .. +31, i.e. tile rows of that lane quarter).
+#pragma once
+
+#include "crc_device.cuh"
+
+namespace crc {
+
+constexpr int pow2ceil_i(int x) {
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+constexpr int imax(int a, int b) { return a > b ? a : b; }
+constexpr int imin(int a, int b) { return a < b ? a : b; }
+
+template <int NH, int H>
+struct RouterCfg {
+    static constexpr int BM = 128;                       // tile rows (TMEM lanes)
+    static constexpr int BK = 64;                        // 64 bf16 = one 128-byte swizzle row
+    static constexpr int NCOL = NH * H;                  // accumulator columns
+    static constexpr int NMMA = NCOL <= 256 ? 1 : 2;     // MMAs per K step (N <= 256 each)
+    static constexpr int NCH = NCOL / NMMA;              // columns per MMA
+    static constexpr int ACC_COLS = pow2ceil_i(imax(32, NCOL));
+    static constexpr int NACC = (2 * ACC_COLS <= 512) ? 2 : 1;   // TMEM double buffering
+    static constexpr int TMEM_COLS = ACC_COLS * NACC;
+    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int B_BYTES = NCOL * BK * 2;
+    static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int STAGES = imin(8, (200 * 1024) / STAGE_BYTES);
+    static constexpr int B_BOX_ROWS = NMMA == 1 ? NCOL : NCH;   // TMA box rows <= 256
+    static constexpr int B_BOXES = NCOL / B_BOX_ROWS;
+    static constexpr uint32_t IDESC = idesc_bf16_f32(BM, NCH);
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+    static constexpr int THREADS = 192;
+
+    static_assert(NH % 16 == 0 && NH >= 16 && NH <= 128, "experts per head");
+    static_assert(NCH % 16 == 0 && NCH >= 16 && NCH <= 256, "MMA N");
+    static_assert(TMEM_COLS <= 512, "TMEM columns");
+    static_assert(STAGES >= 2, "pipeline depth");
+    static_assert((A_BYTES % 1024) == 0 && (B_BYTES % 1024) == 0, "swizzle atom alignment");
+};
+
+struct RouterArgs {
+    float* scores;       // [B][Ts][L][3][NH]
+    uint32_t* err;       // latched device error
+    int B, L, d;
+    int t_begin;         // token coordinate of the first token of this call
+    int T_ext;           // tokens in this call
+    int SB, TB;          // a tile is SB streams x TB tokens
+    int n_sb, n_tb;
+    int num_tiles;       // L * n_sb * n_tb
+    int kblocks;         // ceil(d / 64)
+};
+
+// Softmax of one head, in place: exp(z - max z) / sum, fp32.
+template <int NH>
+__device__ __forceinline__ void head_softmax(float (&z)[NH]) {
+    float m = z[0];
+#pragma unroll
+    for (int i = 1; i < NH; ++i) m = fmaxf(m, z[i]);
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < NH; ++i) {
+        z[i] = __expf(z[i] - m);
+        s += z[i];
+    }
+    const float r = __frcp_rn(s);
+#pragma unroll
+    for (int i = 0; i < NH; ++i) z[i] = z[i] * r;
+}
+
+template <int NH, int H>
+__global__ void __launch_bounds__(192, 1)
+    router_heads_kernel(const __grid_constant__ CUtensorMap tmap_h,
+                        const __grid_constant__ CUtensorMap tmap_w, RouterArgs a) {
+    using Cfg = RouterCfg<NH, H>;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* tiles = smem;
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE_BYTES);
+    uint64_t* empty_bar = full_bar + Cfg::STAGES;
+    uint64_t* tfull_bar = empty_bar + Cfg::STAGES;
+    uint64_t* tempty_bar = tfull_bar + Cfg::NACC;
+    uint64_t* drain_bar = tempty_bar + Cfg::NACC;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < Cfg::STAGES; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], 1);
+        }
+        for (int s = 0; s < Cfg::NACC; ++s) {
+            mbar_init(&tfull_bar[s], 1);
+            mbar_init(&tempty_bar[s], 4);
+        }
+        mbar_init(drain_bar, 1);
+        fence_mbar_init();
+        tma_prefetch_desc(&tmap_h);
+        tma_prefetch_desc(&tmap_w);
+    }
+    if (warp == 1) {
+        tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+    const int tiles_per_layer = a.n_sb * a.n_tb;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA
+        if (lane == 0) {
+            const uint64_t pol_h = l2_evict_first_policy();   // streamed once
+            const uint64_t pol_w = l2_evict_last_policy();    // reused by every tile
+            int stage = 0;
+            uint32_t phase = 0;
+            int issued = 0, failed = 0;
+            for (int tile = blockIdx.x; tile < a.num_tiles && !failed; tile += gridDim.x) {
+                const int l = tile / tiles_per_layer;
+                const int r = tile % tiles_per_layer;
+                const int sb = r / a.n_tb, tb = r % a.n_tb;
+                for (int kb = 0; kb < a.kblocks; ++kb) {
+                    if (!mbar_wait(&empty_bar[stage], phase ^ 1)) {
+                        latch_error(a.err, CRC_ETIMEOUT);
+                        failed = 1;
+                        break;
+                    }
+                    uint8_t* sa = tiles + stage * Cfg::STAGE_BYTES;
+                    uint8_t* sb_ = sa + Cfg::A_BYTES;
+                    mbar_arrive_expect_tx(&full_bar[stage], Cfg::STAGE_BYTES);
+                    tma_load_4d(sa, &tmap_h, &full_bar[stage], kb * Cfg::BK, l,
+                                a.t_begin + tb * a.TB, sb * a.SB, pol_h);
+#pragma unroll
+                    for (int c = 0; c < Cfg::B_BOXES; ++c)
+                        tma_load_3d(sb_ + c * Cfg::B_BOX_ROWS * 128, &tmap_w, &full_bar[stage],
+                                    kb * Cfg::BK, c * Cfg::B_BOX_ROWS, l, pol_w);
+                    ++issued;
+                    if (++stage == Cfg::STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+            }
+            // Never leave with copies in flight: wait for every issued stage to land.
+            int s = stage;
+            uint32_t ph = phase;
+            for (int k = 0; k < imin(issued, Cfg::STAGES); ++k) {
+                if (--s < 0) {
+                    s = Cfg::STAGES - 1;
+                    ph ^= 1;
+                }
+                if (!mbar_wait(&full_bar[s], ph)) latch_error(a.err, CRC_ETIMEOUT);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA
+        if (lane == 0) {
+            int stage = 0, acc = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            int failed = 0;
+            for (int tile = blockIdx.x; tile < a.num_tiles && !failed; tile += gridDim.x) {
+                if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
+                    latch_error(a.err, CRC_ETIMEOUT);
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_tmem = tmem_base + (uint32_t)(acc * Cfg::ACC_COLS);
+                for (int kb = 0; kb < a.kblocks; ++kb) {
+                    if (!mbar_wait(&full_bar[stage], phase)) {
+                        latch_error(a.err, CRC_ETIMEOUT);
+                        failed = 1;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t sa = smem_u32(tiles + stage * Cfg::STAGE_BYTES);
+                    const uint32_t sb_ = sa + Cfg::A_BYTES;
+#pragma unroll
+                    for (int kk = 0; kk < Cfg::BK / 16; ++kk) {
+                        const uint64_t adesc = sw128_kmajor_desc(sa + kk * 32);
+#pragma unroll
+                        for (int c = 0; c < Cfg::NMMA; ++c) {
+                            const uint64_t bdesc =
+                                sw128_kmajor_desc(sb_ + c * Cfg::NCH * 128 + kk * 32);
+                            umma_bf16(d_tmem + c * Cfg::NCH, adesc, bdesc, Cfg::IDESC,
+                                      (kb | kk) != 0);
+                        }
+                    }
+                    umma_commit(&empty_bar[stage]);   // frees the stage when these MMAs finish
+                    if (++stage == Cfg::STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+                if (failed) break;
+                umma_commit(&tfull_bar[acc]);          // accumulator ready for the epilogue
+                if (Cfg::NACC == 2) {
+                    acc ^= 1;
+                    if (acc == 0) acc_phase ^= 1;
+                } else {
+                    acc_phase ^= 1;
+                }
+            }
+            // All issued MMAs must be complete before TMEM is released.
+            umma_commit(drain_bar);
+            if (!mbar_wait(drain_bar, 0)) latch_error(a.err, CRC_ETIMEOUT);
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int quarter = warp & 3;
+        const int row = quarter * 32 + lane;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x) {
+            if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
+                latch_error(a.err, CRC_ETIMEOUT);
+                break;
+            }
+            tc_fence_after();
+            const int l = tile / tiles_per_layer;
+            const int r = tile % tiles_per_layer;
+            const int sb = r / a.n_tb, tb = r % a.n_tb;
+            const int b = sb * a.SB + row / a.TB;
+            const int t = tb * a.TB + row % a.TB;
+            const bool valid = (b < a.B) && (t < a.T_ext);
+            float* out = a.scores + (((size_t)b * a.T_ext + t) * a.L + l) * (size_t)(3 * NH);
+            const uint32_t tbase =
+                tmem_base + (uint32_t)(acc * Cfg::ACC_COLS) + ((uint32_t)(quarter * 32) << 16);
+#pragma unroll 1
+            for (int h = 0; h < H; ++h) {
+                float z[NH];
+#pragma unroll
+                for (int c = 0; c < NH / 16; ++c) {
+                    float part[16];
+                    tmem_ld16(tbase + (uint32_t)(h * NH + c * 16), part);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) z[c * 16 + i] = part[i];
+                }
+                head_softmax<NH>(z);
+                if (valid) {
+                    float4* o = reinterpret_cast<float4*>(out + h * NH);
+#pragma unroll
+                    for (int i = 0; i < NH / 4; ++i)
+                        o[i] = make_float4(z[4 * i], z[4 * i + 1], z[4 * i + 2], z[4 * i + 3]);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+            if (Cfg::NACC == 2) {
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1;
+            } else {
+                acc_phase ^= 1;
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, Cfg::TMEM_COLS);
+    }
+}
+
+}  // namespace crc

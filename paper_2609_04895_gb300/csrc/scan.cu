@@ -1,0 +1,72 @@
+// Host launcher of the cache-scan kernel and the state initialiser.
+#include "cache_scan.cuh"
+#include "crc_internal.h"
+
+namespace crc {
+namespace {
+
+// Writes the header of a state whose bytes were zeroed just before.
+__global__ void state_init_kernel(uint8_t* state, crc_problem p) {
+    StateHeader* h = reinterpret_cast<StateHeader*>(state);
+    h->magic = kStateMagic;
+    h->L = p.L;
+    h->N = p.N;
+    h->K = p.K;
+    h->C = p.C;
+    h->R = p.R;
+    h->B = p.B;
+    h->expert_bytes = p.expert_bytes;
+}
+
+}  // namespace
+
+int launch_state_init(const crc_problem& p, void* state, size_t bytes, cudaStream_t stream) {
+    if (cudaMemsetAsync(state, 0, bytes, stream) != cudaSuccess) return CRC_ECUDA;
+    {
+        ProfScope prof(CRC_KERNEL_STATE, stream);
+        state_init_kernel<<<1, 1, 0, stream>>>(static_cast<uint8_t*>(state), p);
+    }
+    note_launch();
+    return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
+}
+
+template <int V>
+static int launch_scan_t(const crc_problem& p, const float* scores, int T, void* state,
+                         const crc_trace* trace, int trace_T, int trace_t0,
+                         cudaStream_t stream) {
+    ScanArgs a;
+    a.scores = scores;
+    a.state = static_cast<uint8_t*>(state);
+    a.B = p.B;
+    a.T = T;
+    a.L = p.L;
+    a.N = p.N;
+    a.K = p.K;
+    a.C = p.C;
+    a.R = p.R;
+    a.trace_T = trace_T;
+    a.trace_t0 = trace_t0;
+    a.trace_topk = trace ? trace->topk_dev : nullptr;
+    a.trace_miss = trace ? trace->misses_dev : nullptr;
+    a.trace_pro = trace ? trace->proactive_dev : nullptr;
+    const int chains = p.B * p.L;
+    const int warps_per_block = 4;
+    const int grid = (chains + warps_per_block - 1) / warps_per_block;
+    {
+        ProfScope prof(CRC_KERNEL_SCAN, stream);
+        cache_scan_kernel<V><<<grid, 32 * warps_per_block, 0, stream>>>(a);
+    }
+    note_launch();
+    return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
+}
+
+int launch_scan(const crc_problem& p, const float* scores, int T, void* state,
+                const crc_trace* trace, int trace_T, int trace_t0, cudaStream_t stream) {
+    if (T <= 0) return CRC_OK;
+    if (p.N <= 32) return launch_scan_t<1>(p, scores, T, state, trace, trace_T, trace_t0, stream);
+    if (p.N <= 64) return launch_scan_t<2>(p, scores, T, state, trace, trace_T, trace_t0, stream);
+    if (p.N <= 128) return launch_scan_t<4>(p, scores, T, state, trace, trace_T, trace_t0, stream);
+    return launch_scan_t<8>(p, scores, T, state, trace, trace_T, trace_t0, stream);
+}
+
+}  // namespace crc

@@ -1,0 +1,118 @@
+"""Host-only checks of the C-ABI library: it builds, loads, exports every
+symbol include/crc.h declares, and rejects bad arguments before touching the
+GPU (no compute call is made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import crc_synth as S
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def crc():
+    from paper_2609_04895_gb300 import build
+    build.build()
+    from paper_2609_04895_gb300 import crc as C
+    C.load()
+    return C
+
+
+def header_functions():
+    src = open(os.path.join(ROOT, "include", "crc.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(crc_[a-z_]+)\s*\(", src)))
+
+
+def test_every_declared_symbol_is_exported_and_bound(crc):
+    names = header_functions()
+    assert len(names) >= 12
+    lib = crc.load()
+    bound = {n for n, _, _ in crc.EXPORTS}
+    for n in names:
+        assert hasattr(lib, n), n
+        assert n in bound, n
+
+
+def test_struct_layouts_match_header(crc):
+    assert ctypes.sizeof(crc.crc_problem) == 40
+    assert ctypes.sizeof(crc.crc_trace) == 24
+    assert ctypes.sizeof(crc.crc_stats) == 56
+
+
+def test_sizes(crc):
+    p = crc.problem_of(S.QWEN3_30B)
+    B, L, N = p.B, p.L, p.N
+    expect = 256 + B * L * 64 + B * L * N * 4 + 2 * B * N * 4
+    assert crc.crc_state_bytes(p) == (expect + 255) // 256 * 256
+    assert crc.crc_workspace_bytes(p, 16) == B * 16 * L * 3 * N * 4
+    assert crc.crc_workspace_bytes(p, 0) == 0
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("C", 4, 2),        # C < K
+    ("C", 200, 2),      # C > N
+    ("N", 40, 2),       # N % 16 != 0
+    ("K", 40, 2),       # K > 32
+    ("R", 129, 2),      # R > N
+    ("L", 0, 1),
+    ("B", 0, 1),
+    ("reserved", 1, 1),
+])
+def test_problem_validation(crc, field, value, code):
+    p = crc.problem_of(S.QWEN3_30B)
+    setattr(p, field, value)
+    assert crc.crc_state_bytes(p) == 0
+    lib = crc.load()
+    assert lib.crc_state_init(ctypes.byref(p), None, 0, None) == code
+    assert lib.crc_route_scores(ctypes.byref(p), 16, 16, 1, 3, 16, None) == code
+
+
+def test_router_limits_and_pointer_checks(crc):
+    lib = crc.load()
+    p = crc.problem_of(S.QWEN3_30B.with_(N=256, C=32))
+    assert crc.crc_state_bytes(p) > 0                       # the scan takes N = 256
+    assert lib.crc_route_scores(ctypes.byref(p), 16, 16, 1, 3, 16, None) == crc.CRC_EUNSUPPORTED
+    p = crc.problem_of(S.QWEN3_30B)
+    assert lib.crc_route_scores(ctypes.byref(p), 16, 16, 0, 3, 16, None) == crc.CRC_OK   # T = 0
+    assert lib.crc_route_scores(ctypes.byref(p), None, 16, 4, 3, 16, None) == crc.CRC_EINVAL
+    assert lib.crc_route_scores(ctypes.byref(p), 8, 16, 4, 3, 16, None) == crc.CRC_EINVAL
+    assert lib.crc_route_scores(ctypes.byref(p), 16, 16, 4, 4, 16, None) == crc.CRC_EINVAL
+    assert lib.crc_route_scores(ctypes.byref(p), 16, 16, -1, 3, 16, None) == crc.CRC_EINVAL
+    n = crc.crc_state_bytes(p)
+    assert lib.crc_cache_scan(ctypes.byref(p), 16, 4, 256, n - 256, None, None) == crc.CRC_ESTATE
+    assert lib.crc_cache_scan(ctypes.byref(p), 16, 4, 128, n, None, None) == crc.CRC_EINVAL
+    ws = crc.crc_workspace_bytes(p, 1)
+    assert lib.crc_route_and_cache(ctypes.byref(p), 16, 16, 4, 256, n, None, 256, ws - 1,
+                                   None) == crc.CRC_EINVAL
+    assert lib.crc_synth_hidden(1, 1, 1, 3, 0, 0, 0.5, 0.5, None, 16, 16, None) == crc.CRC_EINVAL
+    assert lib.crc_synth_hidden(1, 1, 1, 4, 0, 0, 1.5, 0.5, None, 16, 16, None) == crc.CRC_EINVAL
+
+
+def test_strerror(crc):
+    assert "unsupported" in crc.crc_strerror(2) or "limits" in crc.crc_strerror(2)
+    assert crc.crc_strerror(99) == "unknown error code"
+
+
+def test_product_fails_loudly_without_library(tmp_path):
+    from paper_2609_04895_gb300 import crc as C
+    saved = C._lib
+    try:
+        C._lib = None
+        with pytest.raises(ImportError):
+            C.load(str(tmp_path / "missing.so"))
+    finally:
+        C._lib = saved
+
+
+def test_product_never_imports_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2609_04895_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                txt = open(os.path.join(dirpath, f)).read()
+                assert "import oracle" not in txt and "from oracle" not in txt, f
+                assert "crc_oracle" not in txt, f
