@@ -187,7 +187,7 @@ def test_route_and_cache_equals_pair(C, w):
     for chunk in (1, 7, w.T):
         st = C.State(p)
         tr = C.Trace.alloc(p, w.T)
-        ws = torch.empty(C.crc.crc_workspace_bytes(p, chunk), dtype=torch.uint8, device="cuda")
+        ws = torch.empty(C.crc_workspace_bytes(p, chunk), dtype=torch.uint8, device="cuda")
         C.route_and_cache(p, h, W, st, tr, workspace=ws)
         got = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
         for k in ("cache_bits", "chain_counters", "retention"):
@@ -256,7 +256,7 @@ def test_full_size_workload(C, oracle_lib, w):
     W = host_bits(Wd)
     # the fused call exactly as the benchmark issues it
     chunk = 16
-    ws = torch.empty(C.crc.crc_workspace_bytes(p, chunk), dtype=torch.uint8, device="cuda")
+    ws = torch.empty(C.crc_workspace_bytes(p, chunk), dtype=torch.uint8, device="cuda")
     st = C.State(p)
     tr = C.Trace.alloc(p, w.T)
     C.route_and_cache(p, hd, Wd, st, tr, workspace=ws)
