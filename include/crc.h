@@ -161,6 +161,38 @@ int crc_route_and_cache(const crc_problem *p, const uint16_t *hidden_dev,
                         void *workspace_dev, size_t workspace_bytes, void *stream);
 
 /* ------------------------------------------------------------------------ */
+/* Allocation-free variant (no counterpart in the paper)                    */
+/* ------------------------------------------------------------------------ */
+
+/* Capacity of the library's built-in scratch array, per GPU. */
+#define CRC_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+/* crc_route_and_cache without a workspace argument, for callers that cannot
+ * allocate device memory when they call in: for example code running inside a
+ * serving framework that reserved all device memory for its own pool at
+ * start-up, or a plug-in whose host application forbids allocation after
+ * initialisation (cudaMalloc / cudaFree may also synchronise the whole
+ * device, which a latency-bound decode loop cannot afford).  The caller still
+ * provides every input and output (hidden states, weights, state, trace).
+ * This call allocates nothing: the router scores of each chunk of tokens go
+ * to a fixed array compiled into the library, CRC_NOALLOC_SCRATCH_BYTES bytes
+ * on every GPU where the library is loaded, kept until the process exits.
+ * The chunk is the largest number of tokens whose scores fit in it; a problem
+ * whose scores for one token do not fit (B * L * 3N * 4 bytes above
+ * CRC_NOALLOC_SCRATCH_BYTES) is refused with CRC_EUNSUPPORTED before anything
+ * is enqueued.  The first call on a device looks up that device's copy of the
+ * array (once per device, with the device current); make that first call
+ * before any stream capture.  All calls share the one array per device and
+ * it keeps the last call's contents (nothing in it needs to start at zero:
+ * each chunk's scores are written in full before they are read), so calls
+ * whose kernels may overlap on the GPU -- unordered streams or concurrent
+ * host threads -- race on it: order them.  Results are bit-identical to
+ * crc_route_and_cache. */
+int crc_route_and_cache_noalloc(const crc_problem *p, const uint16_t *hidden_dev,
+                                const uint16_t *w_cat_dev, int32_t T, void *state_dev,
+                                size_t state_bytes, const crc_trace *trace, void *stream);
+
+/* ------------------------------------------------------------------------ */
 /* Support                                                                  */
 /* ------------------------------------------------------------------------ */
 

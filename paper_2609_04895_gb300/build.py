@@ -17,7 +17,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libcrc.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-UNITS = ["api.cu", "router.cu", "scan.cu", "synth.cu"]
+UNITS = ["api.cu", "router.cu", "scan.cu", "synth.cu", "noalloc.cu"]
 
 
 def nvcc() -> str:

@@ -68,6 +68,8 @@ EXPORTS = [
     ("crc_workspace_bytes", SZ, [PP, I32]),
     ("crc_route_and_cache", ctypes.c_int,
      [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P, SZ, P]),
+    ("crc_route_and_cache_noalloc", ctypes.c_int,
+     [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P]),
     ("crc_device_error", ctypes.c_int, []),
     ("crc_launch_count", U64, []),
     ("crc_strerror", ctypes.c_char_p, [ctypes.c_int]),
@@ -175,6 +177,19 @@ def crc_route_and_cache(p: crc_problem, hidden_ptr: int, w_ptr: int, T: int, sta
     _ck(load().crc_route_and_cache(ctypes.byref(p), hidden_ptr, w_ptr, T, state_ptr, state_bytes,
                                    None if trace is None else ctypes.byref(trace), ws_ptr,
                                    ws_bytes, _stream(stream)), "crc_route_and_cache")
+
+
+NOALLOC_SCRATCH_BYTES = 32 << 20
+
+
+def crc_route_and_cache_noalloc(p: crc_problem, hidden_ptr: int, w_ptr: int, T: int,
+                                state_ptr: int, state_bytes: int, trace: crc_trace | None = None,
+                                stream=None):
+    """crc_route_and_cache using the library's built-in scratch array (no workspace)."""
+    _ck(load().crc_route_and_cache_noalloc(ctypes.byref(p), hidden_ptr, w_ptr, T, state_ptr,
+                                           state_bytes,
+                                           None if trace is None else ctypes.byref(trace),
+                                           _stream(stream)), "crc_route_and_cache_noalloc")
 
 
 def crc_device_error() -> int:
