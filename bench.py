@@ -48,6 +48,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--tokens", type=int, default=0,
+                    help="override T (a smaller case, e.g. for an ncu capture)")
+    ap.add_argument("--only", choices=["fused", "router", "scan"], default="fused",
+                    help="time one part alone: router heads or the scan on stored scores")
     return ap.parse_args()
 
 
@@ -268,6 +272,8 @@ def main():
     C = P.crc
 
     w = S.WORKLOADS[args.workload]
+    if args.tokens:
+        w = w.with_(T=args.tokens)
     p = P.problem_of(w)
     heads = 3 if w.R > 0 else 2
     dev = torch.device("cuda", local)
@@ -282,15 +288,26 @@ def main():
     st = P.State(p, device=dev)
     torch.cuda.synchronize()
 
+    if args.only != "fused":
+        scores = P.route_scores(p, hd, Wd, heads=heads)
+        args.no_e2e = True
+
     def step():
+        if args.only == "router":
+            C.crc_route_scores(p, hd.data_ptr(), Wd.data_ptr(), w.T, heads, scores.data_ptr(),
+                               stream)
+            return
         st.init()
+        if args.only == "scan":
+            C.crc_cache_scan(p, scores.data_ptr(), w.T, st.ptr, st.nbytes, None, stream)
+            return
         C.crc_route_and_cache(p, hd.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes, None,
                               ws.data_ptr(), ws.numel(), stream)
 
     for _ in range(max(3, args.warmup)):
         step()
     stats = st.read()
-    assert stats["error"] == 0 and stats["tokens"] == w.T, stats
+    assert stats["error"] == 0 and stats["tokens"] == (0 if args.only == "router" else w.T), stats
     torch.cuda.synchronize()
     if world > 1:
         dist.barrier()
@@ -400,7 +417,7 @@ def main():
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic", "config": workload_config(w, chunk),
+            "data": "synthetic", "config": dict(workload_config(w, chunk), only=args.only),
             "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
             "clocks": clk.summary(),

@@ -12,9 +12,12 @@
 //   UpdateCache: demand-loaded experts fill free slots, then each further one
 //   evicts the lowest-s^T resident outside S (the demand set's order does not
 //   change the resulting set, since inserted experts are in S and protected).
-// Reductions: order-preserving 32-bit keys of the fp32 scores reduced with
-// redux.sync; ties resolved with a ballot (lowest lane = lowest index for an
-// argmax, highest lane = highest index for the last-in-order argmin).
+// Reductions: the fp32 bit patterns of the (non-negative) scores serve as
+// ordered 32-bit keys.  Each lane keeps its keys sorted in policy order, so a
+// warp-wide "first in order" is one redux.sync (max key) and a ballot whose
+// lowest set lane owns it; a "last member" is a lane-local scan, a
+// redux.sync (min key) and a ballot whose highest set lane owns it.  Only the
+// owner lane learns which of its experts was picked.
 #pragma once
 
 #include "crc_device.cuh"
@@ -31,59 +34,83 @@ struct ScanArgs {
     int B, T, L, N, K, C, R;
 };
 
-// Order-preserving key: larger float -> larger unsigned; -0 is mapped to +0.
-// 0 is never produced for a non-NaN input and marks "no element".
-__device__ __forceinline__ uint32_t okey(float x) {
-    uint32_t u = __float_as_uint(x);
-    u = (u == 0x80000000u) ? 0u : u;
-    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-}
+// Keys: scores are non-negative, so their fp32 bit patterns are already
+// ordered like the values; +1 keeps every real key above 0, which marks an
+// empty slot.  Each lane keeps (key, slot) pairs sorted in policy order
+// (key descending, equal keys by ascending slot = ascending expert index).
+__device__ __forceinline__ uint32_t pkey(float x) { return __float_as_uint(x) + 1u; }
 
-// First expert under (score desc, index asc) among eligible ones; -1 if none.
 template <int V>
-__device__ __forceinline__ int warp_argmax(const float (&s)[V], uint32_t elig, int lane,
-                                           uint32_t& key) {
-    uint32_t best = 0u;
-    int bi = 0;
+struct KeyList {
+    uint32_t k[V];
+    uint32_t s[V];
+};
+
+// Stable sort of a lane's V entries: odd-even transposition that swaps only
+// strictly smaller keys forward, so equal keys keep their ascending slots.
+template <int V>
+__device__ __forceinline__ void presort(KeyList<V>& L) {
 #pragma unroll
-    for (int v = 0; v < V; ++v) {
-        const uint32_t k = ((elig >> v) & 1u) ? okey(s[v]) : 0u;
-        if (k > best) {
-            best = k;
-            bi = v;
+    for (int round = 0; round < V; ++round) {
+#pragma unroll
+        for (int j = round & 1; j + 1 < V; j += 2) {
+            const bool sw = L.k[j + 1] > L.k[j];
+            const uint32_t k0 = L.k[j], s0 = L.s[j];
+            L.k[j] = sw ? L.k[j + 1] : k0;
+            L.s[j] = sw ? L.s[j + 1] : s0;
+            L.k[j + 1] = sw ? k0 : L.k[j + 1];
+            L.s[j + 1] = sw ? s0 : L.s[j + 1];
         }
     }
-    const uint32_t m = __reduce_max_sync(kFull, best);
-    key = m;
-    if (m == 0u) return -1;
-    const uint32_t ball = __ballot_sync(kFull, best == m);
-    const int src = __ffs(ball) - 1;
-    return __shfl_sync(kFull, lane * V + bi, src);
 }
 
-// Last expert under (score desc, index asc) among eligible ones, i.e. the
-// smallest score and, among equal scores, the highest index; -1 if none.
+// Removes the warp-wide first entry in policy order: the largest head key and,
+// among lanes whose head has it, the lowest lane (lanes own ascending index
+// ranges; a lane's head is its lowest index among equal keys).  Returns the
+// owner lane (-1 when every list is empty); the owner receives the slot.
 template <int V>
-__device__ __forceinline__ int warp_argmin_last(const float (&s)[V], uint32_t elig, int lane,
-                                                uint32_t& key) {
-    uint32_t best = 0xffffffffu;
-    int bi = -1;
+__device__ __forceinline__ int warp_pop_first(KeyList<V>& L, int lane, uint32_t& key,
+                                              uint32_t& slot) {
+    const uint32_t m = __reduce_max_sync(kFull, L.k[0]);
+    key = m;
+    const uint32_t b = __ballot_sync(kFull, m != 0u && L.k[0] == m);
+    if (b == 0u) return -1;
+    const int owner = __ffs(b) - 1;
+    if (lane == owner) {
+        slot = L.s[0];
+#pragma unroll
+        for (int j = 0; j + 1 < V; ++j) {
+            L.k[j] = L.k[j + 1];
+            L.s[j] = L.s[j + 1];
+        }
+        L.k[V - 1] = 0u;
+    }
+    return owner;
+}
+
+// Last member in policy order among the slots flagged in `members`: smallest
+// key and, among equal keys, the highest index.  Returns the owner lane (-1 if
+// no member); the owner receives the slot.
+template <int V>
+__device__ __forceinline__ int warp_last_member(const uint32_t (&k)[V], uint32_t members,
+                                                int lane, uint32_t& key, uint32_t& slot) {
+    uint32_t best = 0xffffffffu, bs = 0u;
+    bool has = false;
 #pragma unroll
     for (int v = 0; v < V; ++v) {
-        if ((elig >> v) & 1u) {
-            const uint32_t k = okey(s[v]);
-            if (k <= best) {
-                best = k;
-                bi = v;
-            }
+        if (((members >> v) & 1u) && k[v] <= best) {
+            best = k[v];
+            bs = v;
+            has = true;
         }
     }
-    const uint32_t m = __reduce_min_sync(kFull, best);
-    key = m;
-    const uint32_t ball = __ballot_sync(kFull, bi >= 0 && best == m);
-    if (ball == 0u) return -1;
-    const int src = 31 - __clz(ball);
-    return __shfl_sync(kFull, lane * V + bi, src);
+    const uint32_t mn = __reduce_min_sync(kFull, has ? best : 0xffffffffu);
+    key = mn;
+    const uint32_t b = __ballot_sync(kFull, has && best == mn);
+    if (b == 0u) return -1;
+    const int owner = 31 - __clz(b);
+    if (lane == owner) slot = bs;
+    return owner;
 }
 
 template <int V>
@@ -125,58 +152,192 @@ struct ChainRegs {
     uint32_t hits, misses, pro;
 };
 
-// One access at (t, l).  Returns nothing; updates regs and writes the trace.
-template <int V>
+// ---------------------------------------------------------------------------
+// Thread-serial Top-K set of one score row (used for many tokens at once, one
+// token per lane).  A bitonic network on fp32 values (max/min only) finds the
+// K-th largest value theta; a second pass in index order takes every value
+// above theta and, among values equal to theta, the lowest indices -- exactly
+// the first K under (score desc, index asc).
+// ---------------------------------------------------------------------------
+constexpr int pow2_at_least(int x) {
+    int p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+// Sort P values descending (P a power of two), fully unrolled.
+template <int P>
+__device__ __forceinline__ void bitonic_sort_desc(float (&a)[P]) {
+#pragma unroll
+    for (int k = 2; k <= P; k <<= 1) {
+#pragma unroll
+        for (int j = k >> 1; j > 0; j >>= 1) {
+#pragma unroll
+            for (int i = 0; i < P; ++i) {
+                const int l = i ^ j;
+                if (l > i) {
+                    const float hi = fmaxf(a[i], a[l]), lo = fminf(a[i], a[l]);
+                    if ((i & k) == 0) {
+                        a[i] = hi;
+                        a[l] = lo;
+                    } else {
+                        a[i] = lo;
+                        a[l] = hi;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// run <- the P largest of (run, b), both sorted descending; result descending.
+template <int P>
+__device__ __forceinline__ void merge_top_desc(float (&run)[P], const float (&b)[P]) {
+#pragma unroll
+    for (int i = 0; i < P; ++i) run[i] = fmaxf(run[i], b[P - 1 - i]);   // bitonic
+#pragma unroll
+    for (int j = P >> 1; j > 0; j >>= 1) {
+#pragma unroll
+        for (int i = 0; i < P; ++i) {
+            const int l = i ^ j;
+            if (l > i) {
+                const float hi = fmaxf(run[i], run[l]), lo = fminf(run[i], run[l]);
+                run[i] = hi;
+                run[l] = lo;
+            }
+        }
+    }
+}
+
+// Top-K set of row[0..N) (N % 16 == 0, 1 <= K <= min(N, 32), values >= 0) as
+// bits mask[e / 32] bit e % 32; mask must hold N / 32 rounded up words.
+template <int KP>
+__device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, uint32_t* mask) {
+    constexpr int G = KP < 16 ? KP : 16;           // group sorted at once (<= one chunk)
+    float run[KP];
+#pragma unroll
+    for (int i = 0; i < KP; ++i) run[i] = -1.0f;   // below every score
+    for (int c = 0; c < N; c += 16) {
+        float x[16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 f = __ldg(reinterpret_cast<const float4*>(row + c) + q);
+            x[4 * q] = f.x;
+            x[4 * q + 1] = f.y;
+            x[4 * q + 2] = f.z;
+            x[4 * q + 3] = f.w;
+        }
+#pragma unroll
+        for (int g = 0; g < 16; g += G) {
+            float b[KP];
+#pragma unroll
+            for (int i = 0; i < KP; ++i) b[i] = (i < G) ? x[g + i] : -1.0f;
+            bitonic_sort_desc<KP>(b);
+            merge_top_desc<KP>(run, b);
+        }
+    }
+    // theta = K-th largest; `need` of the values equal to theta are taken
+    float theta = run[0];
+#pragma unroll
+    for (int i = 0; i < KP; ++i)
+        if (i == K - 1) theta = run[i];
+    int gt = 0;
+#pragma unroll
+    for (int i = 0; i < KP; ++i)
+        if (i < K && run[i] > theta) ++gt;
+    int need = K - gt;
+    for (int c = 0; c < N; c += 32) {
+        uint32_t w = 0u;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            if (c + 4 * q >= N) break;
+            const float4 f = __ldg(reinterpret_cast<const float4*>(row + c) + q);
+            const float v[4] = {f.x, f.y, f.z, f.w};
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const bool eq = v[u] == theta;
+                const bool take = (v[u] > theta) || (eq && need > 0);
+                need -= eq ? 1 : 0;
+                w |= take ? (1u << (4 * q + u)) : 0u;
+            }
+        }
+        mask[c >> 5] = w;
+    }
+}
+
+// One access at (t, l): refinement, Top-K, misses, UpdateCache.  Updates the
+// chain registers and writes the trace.  ALL_VALID: every lane owns V real
+// experts (N == 32 V), so no validity masks are needed.
+template <int V, bool ALL_VALID>
 __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V],
                                           const float (&pT)[V], const float (&pS)[V],
                                           bool refine, uint32_t valid, int lane, int K, int C,
-                                          int R, uint8_t* topk_out, uint8_t* miss_out,
+                                          int R, bool have_sel, uint32_t sel_in,
+                                          uint8_t* topk_out, uint8_t* miss_out,
                                           uint8_t* pro_out) {
     float sT[V];
 #pragma unroll
     for (int v = 0; v < V; ++v) sT[v] = pR[v] + pT[v];
+    auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
 
     int pro = 0;
     if (refine) {
-        float sST[V];
+        uint32_t kS[V];
+        KeyList<V> A;
 #pragma unroll
-        for (int v = 0; v < V; ++v) sST[v] = cr.aT[v] + pS[v];
-        uint32_t taken = 0u;
-        for (int r = 0; r < R; ++r) {
-            uint32_t ke;
-            const int e = warp_argmax<V>(sST, valid & ~taken, lane, ke);
-            if (e < 0) break;
-            const int owner = e / V;
-            const uint32_t bit = 1u << (e % V);
-            if (lane == owner) taken |= bit;
-            const bool resident = __shfl_sync(kFull, (cr.cache & bit) != 0u, owner);
-            if (resident) continue;
-            if (cr.count < C) {                         // free slot: proactive load
-                if (lane == owner) cr.cache |= bit;
+        for (int v = 0; v < V; ++v) {
+            kS[v] = is_valid(v) ? pkey(cr.aT[v] + pS[v]) : 0u;   // s^ST = a^T + p^S_rho
+            A.k[v] = kS[v];
+            A.s[v] = v;
+        }
+        presort<V>(A);
+        for (int r = 0; r < R; ++r) {                          // candidates, descending
+            uint32_t ke, slot = 0u;
+            const int owner = warp_pop_first<V>(A, lane, ke, slot);
+            if (owner < 0) break;
+            const uint32_t bit = (lane == owner) ? (1u << slot) : 0u;
+            if (__any_sync(kFull, (cr.cache & bit) != 0u)) continue;   // resident
+            if (cr.count < C) {                                // free slot: proactive load
+                cr.cache |= bit;
                 ++cr.count;
                 ++pro;
                 continue;
             }
-            uint32_t kv;
-            const int vic = warp_argmin_last<V>(sST, cr.cache, lane, kv);
-            if (ke > kv) {                              // strictly higher: replace lowest
-                if (lane == vic / V) cr.cache &= ~(1u << (vic % V));
-                if (lane == owner) cr.cache |= bit;
+            uint32_t kv, vslot = 0u;
+            const int vo = warp_last_member<V>(kS, cr.cache, lane, kv, vslot);
+            if (ke > kv) {                                     // strictly higher: replace lowest
+                if (lane == vo) cr.cache &= ~(1u << vslot);
+                cr.cache |= bit;
                 ++pro;
             } else {
-                break;
+                break;                                         // later candidates lose as well
             }
         }
     }
 
-    // native Top-K
-    uint32_t sel = 0u;
+    // native Top-K on p^R: precomputed as a set, or popped in rank order when
+    // the trace wants the order
+    uint32_t sel = sel_in;
     int my_topk = 0;
-    for (int k = 0; k < K; ++k) {
-        uint32_t kk;
-        const int e = warp_argmax<V>(pR, valid & ~sel, lane, kk);
-        if (lane == e / V) sel |= 1u << (e % V);
-        if (lane == k) my_topk = e;
+    const bool want_topk = topk_out != nullptr;
+    if (!have_sel) {
+        KeyList<V> P;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            P.k[v] = is_valid(v) ? pkey(pR[v]) : 0u;
+            P.s[v] = v;
+        }
+        presort<V>(P);
+        sel = 0u;
+        for (int k = 0; k < K; ++k) {
+            uint32_t kk, slot = 0u;
+            const int owner = warp_pop_first<V>(P, lane, kk, slot);
+            if (lane == owner) sel |= 1u << slot;
+            if (want_topk) {
+                const int e = __shfl_sync(kFull, lane * V + (int)slot, owner);
+                if (lane == k) my_topk = e;
+            }
+        }
     }
 
     // demand misses and UpdateCache (Algorithm 1)
@@ -184,13 +345,16 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
     const int nD = (int)__reduce_add_sync(kFull, (uint32_t)__popc(dem));
     const int freeslots = C - cr.count;
     if (nD > freeslots) {
-        uint32_t vset = cr.cache & ~sel;
+        uint32_t kT[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) kT[v] = pkey(sT[v]);
+        uint32_t vset = cr.cache & ~sel;                       // V = C+ \ S
         for (int i = 0; i < nD - freeslots; ++i) {
-            uint32_t kv;
-            const int vic = warp_argmin_last<V>(sT, vset, lane, kv);
-            if (lane == vic / V) {
-                vset &= ~(1u << (vic % V));
-                cr.cache &= ~(1u << (vic % V));
+            uint32_t kv, vslot = 0u;
+            const int vo = warp_last_member<V>(kT, vset, lane, kv, vslot);
+            if (lane == vo) {
+                vset &= ~(1u << vslot);
+                cr.cache &= ~(1u << vslot);
             }
         }
         cr.count = C;
@@ -204,7 +368,7 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
     cr.misses += (uint32_t)nD;
     cr.pro += (uint32_t)pro;
 
-    if (topk_out && lane < K) topk_out[lane] = (uint8_t)my_topk;
+    if (want_topk && lane < K) topk_out[lane] = (uint8_t)my_topk;
     if (lane == 0) {
         if (miss_out) *miss_out = (uint8_t)nD;
         if (pro_out) *pro_out = (uint8_t)pro;
@@ -219,8 +383,10 @@ __device__ __forceinline__ uint32_t lane_bits(const uint32_t* words, int lane, i
     return (words[e0 >> 5] >> (e0 & 31)) & ((1u << V) - 1u);
 }
 
-template <int V>
+template <int V, bool ALL_VALID, int KP>
 __global__ void __launch_bounds__(128) cache_scan_kernel(ScanArgs a) {
+    // Top-K sets of the next 32 tokens of each warp's chain, one row per token
+    __shared__ uint32_t sel_s[4][32][8];
     StateHeader* hdr = reinterpret_cast<StateHeader*>(a.state);
     const StateLayout lay = state_layout(a.B, a.L, a.N);
     ChainState* chains = reinterpret_cast<ChainState*>(a.state + lay.chains);
@@ -269,10 +435,29 @@ __global__ void __launch_bounds__(128) cache_scan_kernel(ScanArgs a) {
         };
         const bool want_s = a.R > 0;
 
+        // Without a trace only the Top-K *set* is needed: it does not depend on
+        // the cache, so lane j computes it for token t + j ahead of the chain.
+        const bool batch_sel = a.trace_topk == nullptr;
+        uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) & 3];
+        const float* row_base = a.scores + ((size_t)b * T * L + l) * row;   // token 0 of chain
+
         Vec<V> cR = load_vec<V>(unit_ptr(0, l), has);
         Vec<V> cT = load_vec<V>(unit_ptr(0, l) + N, has);
         Vec<V> cS = load_vec<V>(pred_ptr(0), has && want_s && (t0 + 0 >= 1));
         for (int t = 0; t < T; ++t) {
+            if (batch_sel && (t & 31) == 0) {
+                __syncwarp();
+                if (t + lane < T) {
+                    const float* r = row_base + (size_t)(t + lane) * L * row;
+                    row_topk_mask<KP>(r, N, a.K, sel_rows[lane]);
+                }
+                __syncwarp();
+            }
+            uint32_t sel_in = 0u;
+            if (batch_sel && has) {
+                const uint32_t e0 = (uint32_t)lane * V;
+                sel_in = (sel_rows[t & 31][e0 >> 5] >> (e0 & 31)) & ((1u << V) - 1u);
+            }
             Vec<V> nR, nT, nS;
             if (t + 1 < T) {
                 nR = load_vec<V>(unit_ptr(t + 1, l), has);
@@ -280,8 +465,8 @@ __global__ void __launch_bounds__(128) cache_scan_kernel(ScanArgs a) {
                 nS = load_vec<V>(pred_ptr(t + 1), has && want_s);
             }
             const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
-            scan_step<V>(cr, cR.v, cT.v, cS.v, want_s && (t0 + t >= 1), valid, lane, a.K, a.C,
-                         a.R, a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
+            scan_step<V, ALL_VALID>(cr, cR.v, cT.v, cS.v, want_s && (t0 + t >= 1), valid, lane, a.K, a.C,
+                         a.R, batch_sel, sel_in, a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
                          a.trace_miss ? a.trace_miss + unit : nullptr,
                          a.trace_pro ? a.trace_pro + unit : nullptr);
             cR = nR;

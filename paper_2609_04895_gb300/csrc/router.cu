@@ -54,6 +54,22 @@ bool make_weight_map(CUtensorMap* m, const uint16_t* w, int L, int N3, int d, in
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// scores [B][T_ext][L][3][NH] fp32 viewed as (NH, 3, L, T, B); a store box is
+// 32 scores x 1 head x 1 layer x TBq tokens x SBq streams (32 rows, 128-byte rows).
+bool make_scores_map(CUtensorMap* m, float* scores, int B, int T_ext, int L, int NH, int TBq,
+                     int SBq) {
+    auto enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[5] = {(cuuint64_t)NH, 3, (cuuint64_t)L, (cuuint64_t)T_ext, (cuuint64_t)B};
+    cuuint64_t strides[4] = {(cuuint64_t)NH * 4, (cuuint64_t)3 * NH * 4,
+                             (cuuint64_t)L * 3 * NH * 4, (cuuint64_t)T_ext * L * 3 * NH * 4};
+    cuuint32_t box[5] = {32, 1, 1, (cuuint32_t)TBq, (cuuint32_t)SBq};
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 5, scores, dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int NH, int H>
 int launch_router_t(const crc_problem& p, const uint16_t* hidden, int T_total, int t_begin,
                     int T_ext, const uint16_t* w_cat, float* scores, uint32_t* err,
@@ -65,6 +81,11 @@ int launch_router_t(const crc_problem& p, const uint16_t* hidden, int T_total, i
     CUtensorMap mh, mw;
     if (!make_hidden_map(&mh, hidden, p.B, T_total, p.L, p.d, TB, SB)) return CRC_ECUDA;
     if (!make_weight_map(&mw, w_cat, p.L, 3 * NH, p.d, Cfg::B_BOX_ROWS)) return CRC_ECUDA;
+    CUtensorMap ms = mh;   // unused when a head is narrower than one 32-score store box
+    if (Cfg::TMA_STORE) {
+        const int TBq = TB < 32 ? TB : 32;
+        if (!make_scores_map(&ms, scores, p.B, T_ext, p.L, NH, TBq, 32 / TBq)) return CRC_ECUDA;
+    }
     RouterArgs a;
     a.scores = scores;
     a.err = err;
@@ -90,7 +111,7 @@ int launch_router_t(const crc_problem& p, const uint16_t* hidden, int T_total, i
     const int grid = a.num_tiles < sm_count() ? a.num_tiles : sm_count();
     {
         ProfScope prof(CRC_KERNEL_ROUTER, stream);
-        router_heads_kernel<NH, H><<<grid, Cfg::THREADS, Cfg::SMEM_BYTES, stream>>>(mh, mw, a);
+        router_heads_kernel<NH, H><<<grid, Cfg::THREADS, Cfg::SMEM_BYTES, stream>>>(mh, mw, ms, a);
     }
     note_launch();
     return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;

@@ -39,11 +39,16 @@ struct RouterCfg {
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = NCOL * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = imin(8, (200 * 1024) / STAGE_BYTES);
+    // Epilogue staging for TMA stores: per epilogue warp two 32 x 32 fp32
+    // tiles (128-byte rows, 128-byte swizzle), used when a head is >= 32 wide.
+    static constexpr bool TMA_STORE = NH >= 32;
+    static constexpr int STAGING_BYTES = TMA_STORE ? 4 * 2 * 4096 : 0;
+    static constexpr int STAGES =
+        imin(8, (232448 - 1024 - 256 - STAGING_BYTES) / STAGE_BYTES);
     static constexpr int B_BOX_ROWS = NMMA == 1 ? NCOL : NCH;   // TMA box rows <= 256
     static constexpr int B_BOXES = NCOL / B_BOX_ROWS;
     static constexpr uint32_t IDESC = idesc_bf16_f32(BM, NCH);
-    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + STAGING_BYTES + 256;
     static constexpr int THREADS = 192;
 
     static_assert(NH % 16 == 0 && NH >= 16 && NH <= 128, "experts per head");
@@ -85,13 +90,16 @@ __device__ __forceinline__ void head_softmax(float (&z)[NH]) {
 template <int NH, int H>
 __global__ void __launch_bounds__(192, 1)
     router_heads_kernel(const __grid_constant__ CUtensorMap tmap_h,
-                        const __grid_constant__ CUtensorMap tmap_w, RouterArgs a) {
+                        const __grid_constant__ CUtensorMap tmap_w,
+                        const __grid_constant__ CUtensorMap tmap_s, RouterArgs a) {
     using Cfg = RouterCfg<NH, H>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* tiles = smem;
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE_BYTES);
+    uint8_t* staging = smem + Cfg::STAGES * Cfg::STAGE_BYTES;          // 1024-aligned
+    uint64_t* full_bar =
+        reinterpret_cast<uint64_t*>(staging + Cfg::STAGING_BYTES);
     uint64_t* empty_bar = full_bar + Cfg::STAGES;
     uint64_t* tfull_bar = empty_bar + Cfg::STAGES;
     uint64_t* tempty_bar = tfull_bar + Cfg::NACC;
@@ -114,6 +122,7 @@ __global__ void __launch_bounds__(192, 1)
         fence_mbar_init();
         tma_prefetch_desc(&tmap_h);
         tma_prefetch_desc(&tmap_w);
+        if (Cfg::TMA_STORE) tma_prefetch_desc(&tmap_s);
     }
     if (warp == 1) {
         tmem_alloc(tmem_slot, Cfg::TMEM_COLS);
@@ -226,6 +235,8 @@ __global__ void __launch_bounds__(192, 1)
         // ------------------------------------------------------------ epilogue
         const int quarter = warp & 3;
         const int row = quarter * 32 + lane;
+        uint8_t* my_stage = staging + (warp - 2) * 2 * 4096;
+        int buf = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x) {
@@ -237,34 +248,64 @@ __global__ void __launch_bounds__(192, 1)
             const int l = tile / tiles_per_layer;
             const int r = tile % tiles_per_layer;
             const int sb = r / a.n_tb, tb = r % a.n_tb;
-            const int b = sb * a.SB + row / a.TB;
-            const int t = tb * a.TB + row % a.TB;
-            const bool valid = (b < a.B) && (t < a.T_ext);
-            float* out = a.scores + (((size_t)b * a.T_ext + t) * a.L + l) * (size_t)(3 * NH);
             const uint32_t tbase =
                 tmem_base + (uint32_t)(acc * Cfg::ACC_COLS) + ((uint32_t)(quarter * 32) << 16);
 #pragma unroll 1
             for (int h = 0; h < H; ++h) {
                 float z[NH];
+                if constexpr (NH >= 32) {
 #pragma unroll
-                for (int c = 0; c < NH / 16; ++c) {
-                    float part[16];
-                    tmem_ld16(tbase + (uint32_t)(h * NH + c * 16), part);
-                    tmem_ld_wait();
+                    for (int c = 0; c < NH / 32; ++c)
+                        tmem_ld32(tbase + (uint32_t)(h * NH + c * 32), z + 32 * c);
+                } else {
+                    tmem_ld16f(tbase + (uint32_t)(h * NH), z);
+                }
+                tmem_ld_wait();
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) z[c * 16 + i] = part[i];
+                for (int c = 0; c < NH / 16; ++c) pin16(z + 16 * c);
+                if (h == H - 1) {             // accumulator fully read: hand it back early
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&tempty_bar[acc]);
                 }
                 head_softmax<NH>(z);
-                if (valid) {
-                    float4* o = reinterpret_cast<float4*>(out + h * NH);
+                if constexpr (Cfg::TMA_STORE) {
+                    // this warp's 32 rows: streams str0.., tokens tok0.. of the scores box
+                    const int row0 = quarter * 32;
+                    const int str0 = sb * a.SB + row0 / a.TB;
+                    const int tok0 = tb * a.TB + row0 % a.TB;
 #pragma unroll
-                    for (int i = 0; i < NH / 4; ++i)
-                        o[i] = make_float4(z[4 * i], z[4 * i + 1], z[4 * i + 2], z[4 * i + 3]);
+                    for (int c = 0; c < NH / 32; ++c) {
+                        uint8_t* sbuf = my_stage + buf * 4096;
+                        buf ^= 1;
+                        if (lane == 0) bulk_wait_read<1>();   // the store that used sbuf is done
+                        __syncwarp();
+                        float4* dst = reinterpret_cast<float4*>(sbuf + lane * 128);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j)
+                            dst[j ^ (lane & 7)] = make_float4(z[32 * c + 4 * j], z[32 * c + 4 * j + 1],
+                                                              z[32 * c + 4 * j + 2],
+                                                              z[32 * c + 4 * j + 3]);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_5d(&tmap_s, sbuf, c * 32, h, l, tok0, str0);
+                            bulk_commit();
+                        }
+                    }
+                } else {
+                    const int b = sb * a.SB + row / a.TB;
+                    const int t = tb * a.TB + row % a.TB;
+                    if (b < a.B && t < a.T_ext) {
+                        float4* o = reinterpret_cast<float4*>(
+                            a.scores + (((size_t)b * a.T_ext + t) * a.L + l) * (size_t)(3 * NH) +
+                            h * NH);
+#pragma unroll
+                        for (int i = 0; i < NH / 4; ++i)
+                            o[i] = make_float4(z[4 * i], z[4 * i + 1], z[4 * i + 2], z[4 * i + 3]);
+                    }
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty_bar[acc]);
             if (Cfg::NACC == 2) {
                 acc ^= 1;
                 if (acc == 0) acc_phase ^= 1;
@@ -272,6 +313,7 @@ __global__ void __launch_bounds__(192, 1)
                 acc_phase ^= 1;
             }
         }
+        if (Cfg::TMA_STORE && lane == 0) bulk_wait<0>();   // every store has landed
     }
 
     tc_fence_before();

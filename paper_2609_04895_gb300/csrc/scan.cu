@@ -30,7 +30,7 @@ int launch_state_init(const crc_problem& p, void* state, size_t bytes, cudaStrea
     return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
 }
 
-template <int V>
+template <int V, bool ALL_VALID, int KP>
 static int launch_scan_t(const crc_problem& p, const float* scores, int T, void* state,
                          const crc_trace* trace, int trace_T, int trace_t0,
                          cudaStream_t stream) {
@@ -54,7 +54,7 @@ static int launch_scan_t(const crc_problem& p, const float* scores, int T, void*
     const int grid = (chains + warps_per_block - 1) / warps_per_block;
     {
         ProfScope prof(CRC_KERNEL_SCAN, stream);
-        cache_scan_kernel<V><<<grid, 32 * warps_per_block, 0, stream>>>(a);
+        cache_scan_kernel<V, ALL_VALID, KP><<<grid, 32 * warps_per_block, 0, stream>>>(a);
     }
     note_launch();
     return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
@@ -63,10 +63,25 @@ static int launch_scan_t(const crc_problem& p, const float* scores, int T, void*
 int launch_scan(const crc_problem& p, const float* scores, int T, void* state,
                 const crc_trace* trace, int trace_T, int trace_t0, cudaStream_t stream) {
     if (T <= 0) return CRC_OK;
-    if (p.N <= 32) return launch_scan_t<1>(p, scores, T, state, trace, trace_T, trace_t0, stream);
-    if (p.N <= 64) return launch_scan_t<2>(p, scores, T, state, trace, trace_T, trace_t0, stream);
-    if (p.N <= 128) return launch_scan_t<4>(p, scores, T, state, trace, trace_T, trace_t0, stream);
-    return launch_scan_t<8>(p, scores, T, state, trace, trace_T, trace_t0, stream);
+#define CRC_SCAN_KP(VV, KPV)                                                              \
+    return (p.N == 32 * VV) ? launch_scan_t<VV, true, KPV>(p, scores, T, state, trace, trace_T,  \
+                                                           trace_t0, stream)                  \
+                            : launch_scan_t<VV, false, KPV>(p, scores, T, state, trace,        \
+                                                            trace_T, trace_t0, stream);
+#define CRC_SCAN(VV)                      \
+    {                                     \
+        if (p.K <= 2) CRC_SCAN_KP(VV, 2)  \
+        if (p.K <= 4) CRC_SCAN_KP(VV, 4)  \
+        if (p.K <= 8) CRC_SCAN_KP(VV, 8)  \
+        if (p.K <= 16) CRC_SCAN_KP(VV, 16) \
+        CRC_SCAN_KP(VV, 32)               \
+    }
+    if (p.N <= 32) CRC_SCAN(1)
+    if (p.N <= 64) CRC_SCAN(2)
+    if (p.N <= 128) CRC_SCAN(4)
+    CRC_SCAN(8)
+#undef CRC_SCAN_KP
+#undef CRC_SCAN
 }
 
 }  // namespace crc

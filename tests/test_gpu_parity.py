@@ -139,6 +139,21 @@ SCAN_CASES = [
 
 
 @pytest.mark.parametrize("name,w,quant", SCAN_CASES, ids=[c[0] for c in SCAN_CASES])
+def test_cache_scan_untraced_state_bit_exact(C, oracle_lib, name, w, quant):
+    # Without a trace the scan takes the Top-K set from its batched selection
+    # instead of rank-ordered pops; the caches and counters must not change.
+    p32 = _oracle_probs32(oracle_lib, w, quant=quant)
+    p = C.problem_of(w)
+    st = C.State(p)
+    C.cache_scan(p, torch.from_numpy(p32).cuda(), st, None)
+    g = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    o = oracle_lib.scan(p32, w.K, w.C, w.R, trace=False)
+    assert np.array_equal(g["cache_bits"], o["cache_bits"])
+    assert np.array_equal(g["chain_counters"], o["counters"])
+    assert np.array_equal(g["retention"].view(np.uint32), o["aT"].view(np.uint32))
+
+
+@pytest.mark.parametrize("name,w,quant", SCAN_CASES, ids=[c[0] for c in SCAN_CASES])
 def test_cache_scan_bit_exact(C, oracle_lib, name, w, quant):
     p32 = _oracle_probs32(oracle_lib, w, quant=quant)
     g = gpu_scan(C, w, p32)
@@ -149,13 +164,21 @@ def test_cache_scan_bit_exact(C, oracle_lib, name, w, quant):
     assert g["error"] == 0 and g["tokens"] == w.T
 
 
-@pytest.mark.parametrize("N,K,C_,R", [(256, 8, 32, 4), (96, 6, 20, 15), (48, 2, 5, 3)])
+@pytest.mark.parametrize("N,K,C_,R", [(256, 8, 32, 4), (96, 6, 20, 15), (48, 2, 5, 3),
+                                      (64, 13, 20, 2), (128, 32, 40, 3), (32, 1, 1, 1)])
 def test_cache_scan_wide_and_odd_n(C, oracle_lib, N, K, C_, R):
     # scan-only sizes the router does not take; probability-like synthetic scores
     w = S.TINY.with_(N=N, K=K, C=C_, R=R, B=3, T=80, L=3)
     p32 = S.near_uniform_scores((w.B, w.T, w.L, 3, N), seed=N)
     g = gpu_scan(C, w, p32)
-    assert_scan_equal(g, oracle_lib.scan(p32, K, C_, R), f"N{N}")
+    o = oracle_lib.scan(p32, K, C_, R)
+    assert_scan_equal(g, o, f"N{N}")
+    p = C.problem_of(w)
+    st = C.State(p)
+    C.cache_scan(p, torch.from_numpy(p32).cuda(), st, None)
+    u = st.read(want_caches=True, want_chain_counters=True)
+    assert np.array_equal(u["cache_bits"], o["cache_bits"])
+    assert np.array_equal(u["chain_counters"], o["counters"])
 
 
 def test_chunked_calls_equal_one_call(C, oracle_lib):
