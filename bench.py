@@ -50,8 +50,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--tokens", type=int, default=0,
                     help="override T (a smaller case, e.g. for an ncu capture)")
-    ap.add_argument("--only", choices=["fused", "router", "scan"], default="fused",
-                    help="time one part alone: router heads or the scan on stored scores")
+    ap.add_argument("--only", choices=["fused", "pair", "router", "scan"], default="fused",
+                    help="fused: crc_route_and_cache as one fused kernel (default); pair: "
+                         "crc_route_scores then crc_cache_scan; router / scan: one part alone")
     return ap.parse_args()
 
 
@@ -284,13 +285,15 @@ def main():
     hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
                            rho_l=w.rho_l, device=dev)
     chunk = args.chunk or w.T
-    ws = torch.empty(C.crc_workspace_bytes(p, chunk), dtype=torch.uint8, device=dev)
+    ws_bytes = (C.crc_fused_workspace_bytes(p) if args.only == "fused" and not args.chunk
+                else C.crc_workspace_bytes(p, chunk))
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     st = P.State(p, device=dev)
     torch.cuda.synchronize()
 
     if args.only != "fused":
         scores = P.route_scores(p, hd, Wd, heads=heads)
-        args.no_e2e = True
+        args.no_e2e = args.no_e2e or args.only != "pair"
 
     def step():
         if args.only == "router":
@@ -299,6 +302,11 @@ def main():
             return
         st.init()
         if args.only == "scan":
+            C.crc_cache_scan(p, scores.data_ptr(), w.T, st.ptr, st.nbytes, None, stream)
+            return
+        if args.only == "pair":
+            C.crc_route_scores(p, hd.data_ptr(), Wd.data_ptr(), w.T, heads, scores.data_ptr(),
+                               stream)
             C.crc_cache_scan(p, scores.data_ptr(), w.T, st.ptr, st.nbytes, None, stream)
             return
         C.crc_route_and_cache(p, hd.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes, None,
@@ -336,27 +344,29 @@ def main():
 
     # roofline of the dominant kernel, timed live over the timed region
     pk, pk_src = peaks()
-    dom = max(("router", "scan"), key=lambda k: kt[k]["ms"])
+    dom = max(("fused", "router", "scan"), key=lambda k: kt[k]["ms"])
     avg_ms = kt[dom]["ms"] / max(1, kt[dom]["launches"])
-    if dom == "router":
+    t_s = kt[dom]["ms"] / 1000.0
+    if dom == "scan":
+        flops = 0.0
+        bytes_ = 4.0 * heads * w.N * w.units * args.steps          # probabilities read once
+        kname = "cache_scan_kernel"
+    elif dom == "router":
         flops = 2.0 * w.d * heads * w.N * w.units * args.steps
-        bytes_ = (2.0 * w.d + 4.0 * heads * w.N) * w.units * args.steps
-        t_s = kt[dom]["ms"] / 1000.0
-        f_frac = flops / t_s / (pk["bf16_tflops"] * 1e12)
-        b_frac = bytes_ / t_s / (pk["hbm_gbs"] * 1e9)
-        if flops / (pk["bf16_tflops"] * 1e12) >= bytes_ / (pk["hbm_gbs"] * 1e9):
-            roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": pk["bf16_tflops"],
-                    "unit": "TFLOP/s", "frac": f_frac}
-        else:
-            roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
-                    "unit": "GB/s", "frac": b_frac}
+        bytes_ = (2.0 * w.d + 4.0 * heads * w.N) * w.units * args.steps   # + scores written
         kname = f"router_heads_kernel<{w.N},{heads}>"
     else:
-        bytes_ = 4.0 * heads * w.N * w.units * args.steps
-        t_s = kt[dom]["ms"] / 1000.0
+        flops, bytes_ = algorithmic(w, w.units, heads)
+        flops, bytes_ = flops * args.steps, bytes_ * args.steps
+        kname = f"fused_route_cache_kernel<{w.N},{heads}>"
+    t_flop = flops / (pk["bf16_tflops"] * 1e12)
+    t_byte = bytes_ / (pk["hbm_gbs"] * 1e9)
+    if t_flop >= t_byte:
+        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": pk["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": t_flop / t_s}
+    else:
         roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
-                "unit": "GB/s", "frac": bytes_ / t_s / (pk["hbm_gbs"] * 1e9)}
-        kname = "cache_scan_kernel"
+                "unit": "GB/s", "frac": t_byte / t_s}
     per_unit, src = committed_traffic(kname, w.name)
     units_per_launch = w.units * args.steps / max(1, kt[dom]["launches"])
     roof["traffic"] = None if per_unit is None else per_unit * units_per_launch
@@ -417,7 +427,10 @@ def main():
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-            "data": "synthetic", "config": dict(workload_config(w, chunk), only=args.only),
+            "data": "synthetic",
+            "config": dict(workload_config(w, None if args.only == "fused" and not args.chunk
+                                           else chunk), path=args.only,
+                           workspace_bytes=int(ws_bytes)),
             "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
             "clocks": clk.summary(),

@@ -148,13 +148,23 @@ int crc_cache_scan(const crc_problem *p, const float *scores_dev, int32_t T,
  * tokens per pass (the router scores of one chunk). */
 size_t crc_workspace_bytes(const crc_problem *p, int32_t chunk_tokens);
 
+/* Workspace bytes with which crc_route_and_cache runs as ONE fused kernel
+ * (router heads on the tensor cores and the scan together; the router scores
+ * then only pass through an L2-sized ring of tiles in the workspace).  The
+ * fused kernel serves calls without a trace and with K <= 8 and 16 <= N <= 128;
+ * other calls, or smaller workspaces, take the chunked two-kernel path.
+ * 0 if p is invalid. */
+size_t crc_fused_workspace_bytes(const crc_problem *p);
+
 /* The whole step: router heads and cache simulation over T tokens, the
  * same results as crc_route_scores followed by crc_cache_scan (bit for bit).
  * hidden_dev bf16 [B][T][L][d]; w_cat_dev bf16 [L][3N][d] (the S head is
- * not computed when R = 0).  The router scores never leave the workspace:
- * workspace_dev holds the scores of one chunk of tokens; the chunk length is
- * the largest that fits in workspace_bytes (at least one token must fit, see
- * crc_workspace_bytes).  256-byte alignment for the workspace. */
+ * not computed when R = 0).  The router scores never leave the workspace.
+ * With workspace_bytes >= crc_fused_workspace_bytes(p) (and no trace, K <= 8)
+ * the call is one fused kernel; otherwise workspace_dev holds the scores of one
+ * chunk of tokens, the chunk length being the largest that fits (at least one
+ * token must fit, see crc_workspace_bytes).  256-byte alignment for the
+ * workspace. */
 int crc_route_and_cache(const crc_problem *p, const uint16_t *hidden_dev,
                         const uint16_t *w_cat_dev, int32_t T, void *state_dev,
                         size_t state_bytes, const crc_trace *trace,
@@ -211,7 +221,7 @@ uint64_t crc_launch_count(void);
  * bookkeeping only; off by default.  Not thread-safe against concurrent
  * library calls from other host threads. */
 enum { CRC_KERNEL_ROUTER = 0, CRC_KERNEL_SCAN = 1, CRC_KERNEL_STATE = 2, CRC_KERNEL_SYNTH = 3,
-       CRC_KERNEL_KINDS = 8 };
+       CRC_KERNEL_FUSED = 4, CRC_KERNEL_KINDS = 8 };
 typedef struct crc_kernel_times {
     uint64_t launches[CRC_KERNEL_KINDS];
     double ms[CRC_KERNEL_KINDS];

@@ -39,7 +39,7 @@ class crc_stats(ctypes.Structure):
                 ("error", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
 
 
-KERNEL_KINDS = {"router": 0, "scan": 1, "state": 2, "synth": 3}
+KERNEL_KINDS = {"router": 0, "scan": 1, "state": 2, "synth": 3, "fused": 4}
 
 
 class crc_kernel_times(ctypes.Structure):
@@ -66,6 +66,7 @@ EXPORTS = [
     ("crc_route_scores", ctypes.c_int, [PP, P, P, I32, I32, P, P]),
     ("crc_cache_scan", ctypes.c_int, [PP, P, I32, P, SZ, ctypes.POINTER(crc_trace), P]),
     ("crc_workspace_bytes", SZ, [PP, I32]),
+    ("crc_fused_workspace_bytes", SZ, [PP]),
     ("crc_route_and_cache", ctypes.c_int,
      [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P, SZ, P]),
     ("crc_route_and_cache_noalloc", ctypes.c_int,
@@ -169,6 +170,10 @@ def crc_cache_scan(p: crc_problem, scores_ptr: int, T: int, state_ptr: int, stat
 
 def crc_workspace_bytes(p: crc_problem, chunk_tokens: int) -> int:
     return int(load().crc_workspace_bytes(ctypes.byref(p), chunk_tokens))
+
+
+def crc_fused_workspace_bytes(p: crc_problem) -> int:
+    return int(load().crc_fused_workspace_bytes(ctypes.byref(p)))
 
 
 def crc_route_and_cache(p: crc_problem, hidden_ptr: int, w_ptr: int, T: int, state_ptr: int,

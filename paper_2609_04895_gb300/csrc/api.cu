@@ -193,6 +193,11 @@ int crc_cache_scan(const crc_problem* p, const float* scores_dev, int32_t T, voi
                        static_cast<cudaStream_t>(stream));
 }
 
+size_t crc_fused_workspace_bytes(const crc_problem* p) {
+    if (check_problem(p, true) != CRC_OK) return 0;
+    return fused_workspace_bytes(*p);
+}
+
 size_t crc_workspace_bytes(const crc_problem* p, int32_t chunk_tokens) {
     if (check_problem(p, true) != CRC_OK || chunk_tokens < 1) return 0;
     return (size_t)p->B * chunk_tokens * p->L * 3 * p->N * sizeof(float);
@@ -210,11 +215,16 @@ int crc_route_and_cache(const crc_problem* p, const uint16_t* hidden_dev,
     if (!hidden_dev || !w_cat_dev || !aligned(hidden_dev, 16) || !aligned(w_cat_dev, 16))
         return CRC_EINVAL;
     if (!workspace_dev || !aligned(workspace_dev, 256)) return CRC_EINVAL;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool traced = trace && (trace->topk_dev || trace->misses_dev || trace->proactive_dev);
+    if (!traced) {
+        rc = launch_fused(*p, hidden_dev, w_cat_dev, T, state_dev, workspace_dev, workspace_bytes, s);
+        if (rc != CRC_EUNSUPPORTED) return rc;
+    }
     const size_t per_token = crc_workspace_bytes(p, 1);
     const long long fit = (long long)(workspace_bytes / per_token);
     if (fit < 1) return CRC_EINVAL;
     const int chunk = fit < T ? (int)fit : T;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     float* scores = static_cast<float*>(workspace_dev);
     const int heads = p->R > 0 ? 3 : 2;
     uint32_t* err = static_cast<uint32_t*>(state_dev) + 1;   // StateHeader::error

@@ -209,14 +209,64 @@ __device__ __forceinline__ void merge_top_desc(float (&run)[P], const float (&b)
     }
 }
 
+// Running top-KP values (descending) of a stream of non-negative scores fed 16
+// at a time; theta(K) is then the K-th largest score and need(K) how many of
+// the scores equal to theta belong to the Top-K set (the lowest indices).
+template <int KP>
+struct TopKAcc {
+    float run[KP];
+    __device__ __forceinline__ void init() {
+#pragma unroll
+        for (int i = 0; i < KP; ++i) run[i] = -1.0f;   // below every score
+    }
+    __device__ __forceinline__ void add16(const float* x) {
+        constexpr int G = KP < 16 ? KP : 16;
+#pragma unroll
+        for (int g = 0; g < 16; g += G) {
+            float b[KP];
+#pragma unroll
+            for (int i = 0; i < KP; ++i) b[i] = (i < G) ? x[g + i] : -1.0f;
+            bitonic_sort_desc<KP>(b);
+            merge_top_desc<KP>(run, b);
+        }
+    }
+    __device__ __forceinline__ float theta(int K) const {
+        float th = run[0];
+#pragma unroll
+        for (int i = 0; i < KP; ++i)
+            if (i == K - 1) th = run[i];
+        return th;
+    }
+    __device__ __forceinline__ int need(int K, float th) const {
+        int gt = 0;
+#pragma unroll
+        for (int i = 0; i < KP; ++i)
+            if (i < K && run[i] > th) ++gt;
+        return K - gt;
+    }
+};
+
+// Threshold pass over 4 consecutive scores: take everything above theta and the
+// first `need` scores equal to theta; returns the 4 bits.
+__device__ __forceinline__ uint32_t take4(float4 f, float th, int& need) {
+    const float v[4] = {f.x, f.y, f.z, f.w};
+    uint32_t w = 0u;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const bool eq = v[u] == th;
+        const bool take = (v[u] > th) || (eq && need > 0);
+        need -= eq ? 1 : 0;
+        w |= take ? (1u << u) : 0u;
+    }
+    return w;
+}
+
 // Top-K set of row[0..N) (N % 16 == 0, 1 <= K <= min(N, 32), values >= 0) as
 // bits mask[e / 32] bit e % 32; mask must hold N / 32 rounded up words.
 template <int KP>
 __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, uint32_t* mask) {
-    constexpr int G = KP < 16 ? KP : 16;           // group sorted at once (<= one chunk)
-    float run[KP];
-#pragma unroll
-    for (int i = 0; i < KP; ++i) run[i] = -1.0f;   // below every score
+    TopKAcc<KP> acc;
+    acc.init();
     for (int c = 0; c < N; c += 16) {
         float x[16];
 #pragma unroll
@@ -227,66 +277,38 @@ __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, ui
             x[4 * q + 2] = f.z;
             x[4 * q + 3] = f.w;
         }
-#pragma unroll
-        for (int g = 0; g < 16; g += G) {
-            float b[KP];
-#pragma unroll
-            for (int i = 0; i < KP; ++i) b[i] = (i < G) ? x[g + i] : -1.0f;
-            bitonic_sort_desc<KP>(b);
-            merge_top_desc<KP>(run, b);
-        }
+        acc.add16(x);
     }
-    // theta = K-th largest; `need` of the values equal to theta are taken
-    float theta = run[0];
-#pragma unroll
-    for (int i = 0; i < KP; ++i)
-        if (i == K - 1) theta = run[i];
-    int gt = 0;
-#pragma unroll
-    for (int i = 0; i < KP; ++i)
-        if (i < K && run[i] > theta) ++gt;
-    int need = K - gt;
+    const float th = acc.theta(K);
+    int need = acc.need(K, th);
     for (int c = 0; c < N; c += 32) {
         uint32_t w = 0u;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
             if (c + 4 * q >= N) break;
-            const float4 f = __ldg(reinterpret_cast<const float4*>(row + c) + q);
-            const float v[4] = {f.x, f.y, f.z, f.w};
-#pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const bool eq = v[u] == theta;
-                const bool take = (v[u] > theta) || (eq && need > 0);
-                need -= eq ? 1 : 0;
-                w |= take ? (1u << (4 * q + u)) : 0u;
-            }
+            w |= take4(__ldg(reinterpret_cast<const float4*>(row + c) + q), th, need) << (4 * q);
         }
         mask[c >> 5] = w;
     }
 }
 
-// One access at (t, l): refinement, Top-K, misses, UpdateCache.  Updates the
-// chain registers and writes the trace.  ALL_VALID: every lane owns V real
-// experts (N == 32 V), so no validity masks are needed.
+// Refinement, access and UpdateCache of one access, given s^T = p^R + p^T,
+// the Spatio prediction of the predecessor and the native Top-K set `sel`
+// (this lane's V bits).  Updates the chain registers; returns the number of
+// proactive loads and writes the demand misses to *n_miss.
 template <int V, bool ALL_VALID>
-__device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V],
-                                          const float (&pT)[V], const float (&pS)[V],
-                                          bool refine, uint32_t valid, int lane, int K, int C,
-                                          int R, bool have_sel, uint32_t sel_in,
-                                          uint8_t* topk_out, uint8_t* miss_out,
-                                          uint8_t* pro_out) {
-    float sT[V];
-#pragma unroll
-    for (int v = 0; v < V; ++v) sT[v] = pR[v] + pT[v];
+__device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V],
+                                          const float (&pS)[V], bool refine, uint32_t valid,
+                                          int lane, int K, int C, int R, uint32_t sel,
+                                          int* n_miss) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
-
     int pro = 0;
     if (refine) {
         uint32_t kS[V];
         KeyList<V> A;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-            kS[v] = is_valid(v) ? pkey(cr.aT[v] + pS[v]) : 0u;   // s^ST = a^T + p^S_rho
+            kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;   // s^ST = a^T + p^S_rho
             A.k[v] = kS[v];
             A.s[v] = v;
         }
@@ -311,31 +333,6 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
                 ++pro;
             } else {
                 break;                                         // later candidates lose as well
-            }
-        }
-    }
-
-    // native Top-K on p^R: precomputed as a set, or popped in rank order when
-    // the trace wants the order
-    uint32_t sel = sel_in;
-    int my_topk = 0;
-    const bool want_topk = topk_out != nullptr;
-    if (!have_sel) {
-        KeyList<V> P;
-#pragma unroll
-        for (int v = 0; v < V; ++v) {
-            P.k[v] = is_valid(v) ? pkey(pR[v]) : 0u;
-            P.s[v] = v;
-        }
-        presort<V>(P);
-        sel = 0u;
-        for (int k = 0; k < K; ++k) {
-            uint32_t kk, slot = 0u;
-            const int owner = warp_pop_first<V>(P, lane, kk, slot);
-            if (lane == owner) sel |= 1u << slot;
-            if (want_topk) {
-                const int e = __shfl_sync(kFull, lane * V + (int)slot, owner);
-                if (lane == k) my_topk = e;
             }
         }
     }
@@ -367,7 +364,49 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
     cr.hits += (uint32_t)(K - nD);
     cr.misses += (uint32_t)nD;
     cr.pro += (uint32_t)pro;
+    *n_miss = nD;
+    return pro;
+}
 
+// One access at (t, l) from the three router probabilities: s^T, the native
+// Top-K (given as a set, or popped in rank order when the trace wants the
+// order), then scan_apply.  Writes the trace.
+template <int V, bool ALL_VALID>
+__device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V],
+                                          const float (&pT)[V], const float (&pS)[V],
+                                          bool refine, uint32_t valid, int lane, int K, int C,
+                                          int R, bool have_sel, uint32_t sel_in,
+                                          uint8_t* topk_out, uint8_t* miss_out,
+                                          uint8_t* pro_out) {
+    auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
+    float sT[V];
+#pragma unroll
+    for (int v = 0; v < V; ++v) sT[v] = __fadd_rn(pR[v], pT[v]);
+
+    uint32_t sel = sel_in;
+    int my_topk = 0;
+    const bool want_topk = topk_out != nullptr;
+    if (!have_sel) {
+        KeyList<V> P;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            P.k[v] = is_valid(v) ? pkey(pR[v]) : 0u;
+            P.s[v] = v;
+        }
+        presort<V>(P);
+        sel = 0u;
+        for (int k = 0; k < K; ++k) {
+            uint32_t kk, slot = 0u;
+            const int owner = warp_pop_first<V>(P, lane, kk, slot);
+            if (lane == owner) sel |= 1u << slot;
+            if (want_topk) {
+                const int e = __shfl_sync(kFull, lane * V + (int)slot, owner);
+                if (lane == k) my_topk = e;
+            }
+        }
+    }
+    int nD;
+    const int pro = scan_apply<V, ALL_VALID>(cr, sT, pS, refine, valid, lane, K, C, R, sel, &nD);
     if (want_topk && lane < K) topk_out[lane] = (uint8_t)my_topk;
     if (lane == 0) {
         if (miss_out) *miss_out = (uint8_t)nD;

@@ -1,6 +1,7 @@
 // Host-side internals shared by the translation units of the library.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -36,6 +37,26 @@ int launch_router(const crc_problem& p, const uint16_t* hidden, int T_total, int
 // [B][trace_T][L][..] and this call writes tokens trace_t0 .. trace_t0 + T - 1.
 int launch_scan(const crc_problem& p, const float* scores, int T, void* state,
                 const crc_trace* trace, int trace_T, int trace_t0, cudaStream_t stream);
+
+// Tensor maps (router.cu): hidden [B][T_total][L][d] as (d, L, T, B) with a
+// 64 x 1 x TB x SB box; W_cat [L][3N][d] as (d, 3N, L) with a 64 x rows x 1 box.
+bool make_hidden_map(CUtensorMap* m, const uint16_t* hidden, int B, int T_total, int L, int d,
+                     int TB, int SB);
+bool make_weight_map(CUtensorMap* m, const uint16_t* w, int L, int N3, int d, int rows);
+
+// Fused route-and-cache (fused_*.cu): workspace bytes that enable it for this
+// problem, and the launch (CRC_EUNSUPPORTED when the problem is outside it).
+size_t fused_workspace_bytes(const crc_problem& p);
+int launch_fused(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                 void* state, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+int launch_fused_n16(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                     void* state, void* workspace, cudaStream_t stream);
+int launch_fused_n32(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                     void* state, void* workspace, cudaStream_t stream);
+int launch_fused_n64(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                     void* state, void* workspace, cudaStream_t stream);
+int launch_fused_n128(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                      void* state, void* workspace, cudaStream_t stream);
 
 int launch_state_init(const crc_problem& p, void* state, size_t bytes, cudaStream_t stream);
 

@@ -1,0 +1,128 @@
+// Host side of the fused route-and-cache kernel: tile plan, workspace layout,
+// tensor maps and the cooperative launch (all CTAs resident at once, which the
+// kernel's producer / consumer waits rely on).
+#pragma once
+
+#include <algorithm>
+
+#include "crc_internal.h"
+#include "fused.cuh"
+
+namespace crc {
+
+struct FusedPlan {
+    int SB, TB, n_bg, n_tb, tiles_per_tb, num_tiles, ring, n_items;
+    size_t slot_bytes, ctl_bytes, total;
+};
+
+// Tile = SB streams x TB tokens of one layer, TB as long as the call allows
+// (128 tokens of one stream when T >= 128).  Tiles go in the order (token
+// block, layer, stream group), so a layer's weights are fetched once per
+// token block; the ring holds three token blocks of records.  T = 0 gives the
+// largest layout.
+inline FusedPlan fused_plan(const crc_problem& p, int T) {
+    FusedPlan f;
+    int tb = 128;
+    if (T > 0)
+        while (tb > 1 && tb / 2 >= T) tb >>= 1;
+    f.TB = tb;
+    f.SB = 128 / tb;
+    f.n_bg = (p.B + f.SB - 1) / f.SB;
+    f.tiles_per_tb = p.L * f.n_bg;
+    f.n_tb = (T + f.TB - 1) / f.TB;
+    f.num_tiles = f.n_tb * f.tiles_per_tb;
+    f.ring = 3 * f.tiles_per_tb;
+    if (T > 0) f.ring = std::min(f.ring, f.num_tiles);
+    f.n_items = f.n_tb * p.L * p.B;
+    const int NW = (p.N + 31) / 32;
+    f.slot_bytes = (size_t)128 * 4 * (NW + p.N * (p.R > 0 ? 2 : 1));
+    const size_t ctl = 256 + (size_t)4 * 3 * f.tiles_per_tb * 2 + (size_t)4 * p.B * p.L;
+    f.ctl_bytes = (ctl + 255) & ~(size_t)255;
+    f.total = f.ctl_bytes + (size_t)3 * f.tiles_per_tb * f.slot_bytes;
+    return f;
+}
+
+template <int NH, int H, int V, bool ALL_VALID, int KP>
+int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                   void* state, void* workspace, cudaStream_t stream) {
+    using Cfg = FusedCfg<NH, H>;
+    using RC = typename Cfg::RC;
+    const FusedPlan f = fused_plan(p, T);
+    CUtensorMap mh, mw;
+    if (!make_hidden_map(&mh, hidden, p.B, T, p.L, p.d, f.TB, f.SB)) return CRC_ECUDA;
+    if (!make_weight_map(&mw, w_cat, p.L, 3 * NH, p.d, RC::B_BOX_ROWS)) return CRC_ECUDA;
+    auto kern = fused_route_cache_kernel<NH, H, V, ALL_VALID, KP>;
+    static bool attr_set = false;
+    if (!attr_set) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 Cfg::SMEM_BYTES) != cudaSuccess)
+            return CRC_ECUDA;
+        attr_set = true;
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Cfg::THREADS,
+                                                      Cfg::SMEM_BYTES) != cudaSuccess ||
+        per_sm < 1)
+        return CRC_EUNSUPPORTED;
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    if (cudaMemsetAsync(ws, 0, f.ctl_bytes, stream) != cudaSuccess) return CRC_ECUDA;
+    FusedArgs a;
+    a.state = static_cast<uint8_t*>(state);
+    a.B = p.B;
+    a.L = p.L;
+    a.N = p.N;
+    a.K = p.K;
+    a.C = p.C;
+    a.R = p.R;
+    a.T = T;
+    a.SB = f.SB;
+    a.TB = f.TB;
+    a.n_bg = f.n_bg;
+    a.n_tb = f.n_tb;
+    a.tiles_per_tb = f.tiles_per_tb;
+    a.num_tiles = f.num_tiles;
+    a.ring = f.ring;
+    a.kblocks = (p.d + RC::BK - 1) / RC::BK;
+    a.n_items = f.n_items;
+    a.ctl = reinterpret_cast<uint32_t*>(ws);
+    a.tile_done = reinterpret_cast<uint32_t*>(ws + 256);
+    a.readers = a.tile_done + f.ring;
+    a.prog = a.readers + f.ring;
+    a.ring_base = ws + f.ctl_bytes;
+    a.slot_bytes = f.slot_bytes;
+    void* args[] = {(void*)&mh, (void*)&mw, (void*)&a};
+    const int grid = sm_count();
+    cudaError_t e;
+    {
+        ProfScope prof(CRC_KERNEL_FUSED, stream);
+        e = cudaLaunchCooperativeKernel((const void*)kern, grid, Cfg::THREADS, args,
+                                        Cfg::SMEM_BYTES, stream);
+    }
+    note_launch();
+    return e == cudaSuccess ? CRC_OK : CRC_ECUDA;
+}
+
+// Dispatch on heads (R > 0 needs the Spatio head) and the Top-K network width.
+template <int NH, int V, bool ALL_VALID>
+int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat,
+                       int T, void* state, void* workspace, cudaStream_t stream) {
+#define CRC_FUSED_KP(HV)                                                                      \
+    if (p.K <= 2)                                                                             \
+        return launch_fused_t<NH, HV, V, ALL_VALID, 2>(p, hidden, w_cat, T, state, workspace, \
+                                                       stream);                               \
+    if (p.K <= 4)                                                                             \
+        return launch_fused_t<NH, HV, V, ALL_VALID, 4>(p, hidden, w_cat, T, state, workspace, \
+                                                       stream);                               \
+    if (p.K <= 8)                                                                             \
+        return launch_fused_t<NH, HV, V, ALL_VALID, 8>(p, hidden, w_cat, T, state, workspace, \
+                                                       stream);                               \
+    return CRC_EUNSUPPORTED;
+    if (p.R > 0) {
+        CRC_FUSED_KP(3)
+    } else {
+        CRC_FUSED_KP(2)
+    }
+#undef CRC_FUSED_KP
+}
+
+}  // namespace crc

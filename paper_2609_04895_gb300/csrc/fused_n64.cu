@@ -1,0 +1,11 @@
+// Fused route-and-cache instantiations for N = 64 experts per layer.
+#include "fused_launch.cuh"
+
+namespace crc {
+
+int launch_fused_n64(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                     void* state, void* workspace, cudaStream_t stream) {
+    return launch_fused_for_n<64, 2, true>(p, hidden, w_cat, T, state, workspace, stream);
+}
+
+}  // namespace crc

@@ -7,7 +7,6 @@
 #include "router_gemm.cuh"
 
 namespace crc {
-namespace {
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -69,6 +68,8 @@ bool make_scores_map(CUtensorMap* m, float* scores, int B, int T_ext, int L, int
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
+
+namespace {
 
 template <int NH, int H>
 int launch_router_t(const crc_problem& p, const uint16_t* hidden, int T_total, int t_begin,

@@ -84,7 +84,7 @@ __device__ __forceinline__ void head_softmax(float (&z)[NH]) {
     }
     const float r = __frcp_rn(s);
 #pragma unroll
-    for (int i = 0; i < NH; ++i) z[i] = z[i] * r;
+    for (int i = 0; i < NH; ++i) z[i] = __fmul_rn(z[i], r);
 }
 
 template <int NH, int H>

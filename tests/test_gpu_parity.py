@@ -303,6 +303,18 @@ def test_full_size_workload(C, oracle_lib, w):
         ref = oracle_lib.unit_probs(row, W[l], w.N, H=heads)
         assert rel_err(scores[b, t, l, :heads].cpu().numpy(), ref).max() <= TOL
 
+    # the fused kernel (no trace, fused workspace) equals the chunked call on every chain
+    wsf = torch.empty(C.crc_fused_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    stf = C.State(p)
+    C.crc_profile_begin()
+    C.route_and_cache(p, hd, Wd, stf, None, workspace=wsf)
+    assert C.crc_profile_end()["fused"]["launches"] == 1
+    fz = stf.read(want_caches=True, want_chain_counters=True)
+    assert fz["error"] == 0 and fz["tokens"] == w.T
+    assert np.array_equal(fz["cache_bits"], fused["cache_bits"])
+    assert np.array_equal(fz["chain_counters"], fused["chain_counters"])
+    del wsf
+
     # fused == pair on every stream
     st2 = C.State(p)
     tr2 = C.Trace.alloc(p, w.T)
@@ -330,3 +342,43 @@ def test_full_size_workload(C, oracle_lib, w):
     assert np.array_equal(g["cache_bits"][b], o["cache_bits"][0])
     assert np.array_equal(g["retention"][b].view(np.uint32), o["aT"][0].view(np.uint32))
     assert np.array_equal(g["chain_counters"][b], o["counters"][0])
+
+
+# --------------------------------------------------------------------------- #
+FUSED_CASES = [
+    ("tiny", S.TINY),                                               # SB=4, TB=32
+    ("qwen3", S.QWEN3_30B.with_(T=41, L=5)),                        # SB=32, TB=4, ragged T
+    ("gptoss", S.GPT_OSS_20B.with_(B=128, T=23, L=3, d=576)),       # 4 stream groups
+    ("r0", S.QWEN3_30B.with_(B=40, T=19, L=4, R=0, C=16)),          # 2 heads, partial group
+    ("n64-one-layer", S.TINY.with_(N=64, K=3, C=9, R=5, B=6, T=50, L=1, d=192)),
+    ("k1", S.TINY.with_(K=1, C=2, R=2, B=9, T=33)),
+]
+
+
+@pytest.mark.parametrize("name,w", FUSED_CASES, ids=[c[0] for c in FUSED_CASES])
+def test_fused_kernel_equals_pair(C, name, w):
+    """route_and_cache with a workspace large enough for the fused kernel (no
+    trace) equals route_scores + cache_scan bit for bit, over two calls that
+    continue the same streams."""
+    p = C.problem_of(w)
+    W = dev_bf16(S.weights(w, seed=31))
+    h = dev_bf16(S.hidden(w, seed=32))
+    heads = 3 if w.R > 0 else 2
+    split = [w.T // 3, w.T - w.T // 3]
+    st_pair, st_fused = C.State(p), C.State(p)
+    ws = torch.empty(C.crc_fused_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    t0 = 0
+    for n in split:
+        hc = h[:, t0:t0 + n].contiguous()
+        C.cache_scan(p, C.route_scores(p, hc, W, heads=heads), st_pair)
+        C.crc_profile_begin()
+        C.route_and_cache(p, hc, W, st_fused, None, workspace=ws)
+        kt = C.crc_profile_end()
+        assert kt["fused"]["launches"] == 1 and kt["router"]["launches"] == 0
+        t0 += n
+    a = st_pair.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    b = st_fused.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    assert b["error"] == 0 and b["tokens"] == w.T
+    for k in ("cache_bits", "chain_counters"):
+        assert np.array_equal(a[k], b[k]), k
+    assert np.array_equal(a["retention"].view(np.uint32), b["retention"].view(np.uint32))
