@@ -126,6 +126,14 @@ __device__ __forceinline__ void tmem_cols(uint32_t taddr, float* z) {
     }
 }
 template <int CW>
+__device__ __forceinline__ void tmem_put(uint32_t taddr, const float* z) {
+    if constexpr (CW == 32) {
+        tmem_st32(taddr, z);
+    } else {
+        tmem_st16(taddr, z);
+    }
+}
+template <int CW>
 __device__ __forceinline__ void pin_cols(float* z) {
 #pragma unroll
     for (int c = 0; c < CW / 16; ++c) pin16(z + 16 * c);
@@ -363,14 +371,21 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
                     for (int i = 0; i < CW; ++i) m = fmaxf(m, z[i]);
                 }
+                // each exp(z - max) is computed once and parked in the
+                // accumulator's own TMEM columns for the normalising pass
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
 #pragma unroll
-                    for (int i = 0; i < CW; ++i) s += __expf(z[i] - m);
+                    for (int i = 0; i < CW; ++i) {
+                        z[i] = __expf(z[i] - m);
+                        s += z[i];
+                    }
+                    tmem_put<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                 }
+                tmem_st_wait();
                 const float r = __frcp_rn(s);
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
@@ -381,10 +396,9 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
                         for (int q = 0; q < CW / 4; ++q)
                             pS_p[(size_t)(c * CW / 4 + q) * 128 + row] =
-                                make_float4(__fmul_rn(__expf(z[4 * q] - m), r),
-                                            __fmul_rn(__expf(z[4 * q + 1] - m), r),
-                                            __fmul_rn(__expf(z[4 * q + 2] - m), r),
-                                            __fmul_rn(__expf(z[4 * q + 3] - m), r));
+                                make_float4(__fmul_rn(z[4 * q], r), __fmul_rn(z[4 * q + 1], r),
+                                            __fmul_rn(z[4 * q + 2], r),
+                                            __fmul_rn(z[4 * q + 3], r));
                     }
                 }
             }
@@ -413,10 +427,15 @@ __global__ void __launch_bounds__(512, 1)
                 pin_cols<CW>(y);
 #pragma unroll
                 for (int i = 0; i < CW; ++i) {
-                    sR += __expf(z[i] - mR);
-                    sTs += __expf(y[i] - mT);
+                    z[i] = __expf(z[i] - mR);
+                    y[i] = __expf(y[i] - mT);
+                    sR += z[i];
+                    sTs += y[i];
                 }
+                tmem_put<CW>(tbase + (uint32_t)(c * CW), z);
+                tmem_put<CW>(tbase + (uint32_t)(NH + c * CW), y);
             }
+            tmem_st_wait();
             const float rR = __frcp_rn(sR), rT = __frcp_rn(sTs);
             TopKAcc<KP> topk;
             topk.init();
@@ -431,8 +450,8 @@ __global__ void __launch_bounds__(512, 1)
                 for (int i = 0; i < CW; ++i) {
                     // separately rounded products and sum (no contraction into an
                     // FMA), exactly as the router writes p^R, p^T and the scan adds them
-                    z[i] = __fmul_rn(__expf(z[i] - mR), rR);                 // p^R
-                    y[i] = __fadd_rn(z[i], __fmul_rn(__expf(y[i] - mT), rT));  // s^T
+                    z[i] = __fmul_rn(z[i], rR);                  // p^R
+                    y[i] = __fadd_rn(z[i], __fmul_rn(y[i], rT));  // s^T
                 }
                 if (ok) {
 #pragma unroll
@@ -458,10 +477,9 @@ __global__ void __launch_bounds__(512, 1)
                 }
 #pragma unroll
                 for (int q = 0; q < CW / 4; ++q) {
-                    const float4 f = make_float4(__fmul_rn(__expf(z[4 * q] - mR), rR),
-                                                 __fmul_rn(__expf(z[4 * q + 1] - mR), rR),
-                                                 __fmul_rn(__expf(z[4 * q + 2] - mR), rR),
-                                                 __fmul_rn(__expf(z[4 * q + 3] - mR), rR));
+                    const float4 f = make_float4(__fmul_rn(z[4 * q], rR), __fmul_rn(z[4 * q + 1], rR),
+                                                 __fmul_rn(z[4 * q + 2], rR),
+                                                 __fmul_rn(z[4 * q + 3], rR));
                     word |= take4(f, th, need) << ((c * CW + 4 * q) & 31);
                 }
                 if (((c + 1) * CW) % 32 == 0 || c == NCHK - 1) {
@@ -555,24 +573,21 @@ __global__ void __launch_bounds__(512, 1)
             const uint8_t* prv =
                 k_prev >= 0 ? a.ring_base + (size_t)(k_prev % a.ring) * a.slot_bytes : nullptr;
             const float* carry_in = carry + ((size_t)parity * a.B + b) * N + e0;
-            int last_row = -1;
-            for (int tbi = 0; tbi < a.TB; ++tbi) {
-                const int t = tb * a.TB + tbi;
-                if (t >= a.T) break;
+            const int steps = imin(a.TB, a.T - tb * a.TB);
+            const int last_row = sbi * a.TB + steps - 1;
+            // inputs of step tbi: s^T, the Top-K bits and p^S of the predecessor
+            auto fetch = [&](int tbi, float (&sT)[V], float (&pS)[V], uint32_t& sel) {
                 const int r = sbi * a.TB + tbi;
-                last_row = r;
-                float sT[V], pS[V];
 #pragma unroll
                 for (int v = 0; v < V; ++v) sT[v] = pS[v] = 0.f;
-                if (has) ring_vec<V>(own + RL::ST, lane, r, sT);
-                uint32_t sel = 0u;
-                if (has)
-                    sel = (__ldcg(reinterpret_cast<const uint32_t*>(own + RL::SEL) +
-                                  (size_t)(e0 >> 5) * 128 + r) >>
-                           (e0 & 31)) &
-                          ((1u << V) - 1u);
-                const bool refine = want_s && (t0g + t >= 1);
-                if (refine && has) {
+                sel = 0u;
+                if (!has) return;
+                ring_vec<V>(own + RL::ST, lane, r, sT);
+                sel = (__ldcg(reinterpret_cast<const uint32_t*>(own + RL::SEL) +
+                              (size_t)(e0 >> 5) * 128 + r) >>
+                       (e0 & 31)) &
+                      ((1u << V) - 1u);
+                if (want_s && (t0g + tb * a.TB + tbi >= 1)) {
                     if (l > 0) {
                         ring_vec<V>(psl + RL::PS, lane, r, pS);
                     } else if (tbi > 0) {
@@ -585,11 +600,45 @@ __global__ void __launch_bounds__(512, 1)
                         for (int v = 0; v < V; ++v) pS[v] = x.v[v];
                     }
                 }
+            };
+            // Pull the next 128-byte lines of this lane's chunks into L2 ahead of
+            // use (rows r .. r+7 of a chunk share one line; sel words 32 rows).
+            auto prefetch_rows = [&](int tbi) {
+                if (!has || tbi >= steps) return;
+                const int r = sbi * a.TB + tbi;
+                const int ch = (int)(e0 >> 2);
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(own + RL::ST +
+                                                               ((size_t)ch * 128 + r) * 16));
+                if (want_s)
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(psl + RL::PS +
+                                                                   ((size_t)ch * 128 + r) * 16));
+                if ((tbi & 31) == 0)
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(
+                        own + RL::SEL + ((size_t)(e0 >> 5) * 128 + r) * 4));
+            };
+            prefetch_rows(8);
+            prefetch_rows(16);
+            float cT[V], cS[V];
+            uint32_t csel;
+            fetch(0, cT, cS, csel);
+            for (int tbi = 0; tbi < steps; ++tbi) {
+                float nT[V], nS[V];
+                uint32_t nsel = 0u;
+                if (tbi + 1 < steps) fetch(tbi + 1, nT, nS, nsel);
+                if ((tbi & 7) == 0) prefetch_rows(tbi + 24);
+                const bool refine = want_s && (t0g + tb * a.TB + tbi >= 1);
                 int nD;
-                scan_apply<V, ALL_VALID>(cr, sT, pS, refine, valid, lane, a.K, a.C, a.R, sel, &nD);
+                scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R, csel,
+                                         &nD);
+#pragma unroll
+                for (int v = 0; v < V; ++v) {
+                    cT[v] = nT[v];
+                    cS[v] = nS[v];
+                }
+                csel = nsel;
             }
             // the last layer hands p^S of the call's last token to layer 0 of the next call
-            if (l == L - 1 && want_s && tb * a.TB + a.TB >= a.T && last_row >= 0 && has) {
+            if (l == L - 1 && want_s && tb * a.TB + a.TB >= a.T && steps > 0 && has) {
                 float pl[V];
                 ring_vec<V>(own + RL::PS, lane, last_row, pl);   // has: lane owns experts
                 float* dst = carry + ((size_t)(parity ^ 1u) * a.B + b) * N + e0;
