@@ -437,6 +437,11 @@ __global__ void __launch_bounds__(512, 1)
             }
             tmem_st_wait();
             const float rR = __frcp_rn(sR), rT = __frcp_rn(sTs);
+            // With a single accumulator, p^R is parked in the spare TMEM columns
+            // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
+            // before the Top-K selection runs.
+            constexpr bool PARK = RC::NACC == 1 && RC::NCOL + NH <= RC::ACC_COLS;
+            const uint32_t pbase = tbase + (uint32_t)RC::NCOL;
             TopKAcc<KP> topk;
             topk.init();
 #pragma unroll 1
@@ -459,27 +464,51 @@ __global__ void __launch_bounds__(512, 1)
                         sT_p[(size_t)(c * CW / 4 + q) * 128 + row] =
                             make_float4(y[4 * q], y[4 * q + 1], y[4 * q + 2], y[4 * q + 3]);
                 }
+                if constexpr (PARK) {
+                    tmem_put<CW>(pbase + (uint32_t)(c * CW), z);
+                } else {
 #pragma unroll
-                for (int g = 0; g < CW; g += 16) topk.add16(z + g);
+                    for (int g = 0; g < CW; g += 16) topk.add16(z + g);
+                }
+            }
+            if constexpr (PARK) {
+                tmem_st_wait();
+                tc_fence_before();                        // accumulator columns fully read
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+#pragma unroll 1
+                for (int c = 0; c < NCHK; ++c) {
+                    tmem_cols<CW>(pbase + (uint32_t)(c * CW), z);
+                    tmem_ld_wait();
+                    pin_cols<CW>(z);
+#pragma unroll
+                    for (int g = 0; g < CW; g += 16) topk.add16(z + g);
+                }
             }
             const float th = topk.theta(a.K);
             int need = topk.need(a.K, th);
             uint32_t word = 0u;
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
-                tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
-                tmem_ld_wait();
-                pin_cols<CW>(z);
-                if (c == NCHK - 1) {                      // accumulator fully read
-                    tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+                if constexpr (PARK) {
+                    tmem_cols<CW>(pbase + (uint32_t)(c * CW), z);
+                    tmem_ld_wait();
+                    pin_cols<CW>(z);
+                } else {
+                    tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
+                    tmem_ld_wait();
+                    pin_cols<CW>(z);
+                    if (c == NCHK - 1) {                  // accumulator fully read
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+                    }
+#pragma unroll
+                    for (int i = 0; i < CW; ++i) z[i] = __fmul_rn(z[i], rR);   // p^R
                 }
 #pragma unroll
                 for (int q = 0; q < CW / 4; ++q) {
-                    const float4 f = make_float4(__fmul_rn(z[4 * q], rR), __fmul_rn(z[4 * q + 1], rR),
-                                                 __fmul_rn(z[4 * q + 2], rR),
-                                                 __fmul_rn(z[4 * q + 3], rR));
+                    const float4 f = make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
                     word |= take4(f, th, need) << ((c * CW + 4 * q) & 31);
                 }
                 if (((c + 1) * CW) % 32 == 0 || c == NCHK - 1) {
