@@ -305,15 +305,27 @@ __device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V]
     int pro = 0;
     if (refine) {
         uint32_t kS[V];
-        KeyList<V> A;
+        uint32_t u = 0u;                                       // best key outside the cache
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;   // s^ST = a^T + p^S_rho
+            if (!((cr.cache >> v) & 1u)) u = kS[v] > u ? kS[v] : u;
+        }
+        // When at least R experts score strictly above every non-resident one,
+        // the first R candidates are all resident and the pass changes nothing.
+        const uint32_t u1 = __reduce_max_sync(kFull, u);
+        uint32_t above = 0u;
+#pragma unroll
+        for (int v = 0; v < V; ++v) above += kS[v] > u1 ? 1u : 0u;
+        const bool idle = u1 == 0u || (int)__reduce_add_sync(kFull, above) >= R;
+        KeyList<V> A;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
             A.k[v] = kS[v];
             A.s[v] = v;
         }
-        presort<V>(A);
-        for (int r = 0; r < R; ++r) {                          // candidates, descending
+        if (!idle) presort<V>(A);
+        for (int r = 0; r < (idle ? 0 : R); ++r) {            // candidates, descending
             uint32_t ke, slot = 0u;
             const int owner = warp_pop_first<V>(A, lane, ke, slot);
             if (owner < 0) break;
