@@ -48,6 +48,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--capacity", type=int, default=0,
+                    help="cache slots C per (stream, layer) (0 = the workload's; the sweep takes 16/32/64/96)")
+    ap.add_argument("--proactive", type=int, default=None,
+                    help="proactive-load bound R (default: the workload's; the large shape takes 2 or 8)")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override T (a smaller case, e.g. for an ncu capture)")
     ap.add_argument("--only", choices=["fused", "pair", "router", "scan"], default="fused",
@@ -212,11 +216,22 @@ def cpu_oracle_sample(w, seconds: float):
                       f"(fp64 router heads + literal scan), {dt:.1f} s wall"}, units, dt
 
 
+def workload_of(args):
+    w = S.WORKLOADS[args.workload]
+    if args.tokens:
+        w = w.with_(T=args.tokens)
+    if args.capacity:
+        w = w.with_(C=args.capacity)
+    if args.proactive is not None:
+        w = w.with_(R=args.proactive)
+    return w
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    w = S.WORKLOADS[args.workload]
+    w = workload_of(args)
     import oracle
     oracle.build()
     threads = oracle.default_threads()
@@ -272,13 +287,13 @@ def main():
     import paper_2609_04895_gb300 as P
     C = P.crc
 
-    w = S.WORKLOADS[args.workload]
-    if args.tokens:
-        w = w.with_(T=args.tokens)
+    w = workload_of(args)
     p = P.problem_of(w)
     heads = 3 if w.R > 0 else 2
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream()
+    if 2 * w.B * w.T * w.L * w.d > STREAM_BYTES:
+        return run_streamed(args, P, C, w, p, heads, dev, stream, rank, world)
 
     # inputs, resident in HBM before timing (untimed generation)
     Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
@@ -342,80 +357,14 @@ def main():
     units_all = w.units * world
     value = units_all / (ms_per_step / 1000.0)
 
-    # roofline of the dominant kernel, timed live over the timed region
-    pk, pk_src = peaks()
-    dom = max(("fused", "router", "scan"), key=lambda k: kt[k]["ms"])
-    avg_ms = kt[dom]["ms"] / max(1, kt[dom]["launches"])
-    t_s = kt[dom]["ms"] / 1000.0
-    if dom == "scan":
-        flops = 0.0
-        bytes_ = 4.0 * heads * w.N * w.units * args.steps          # probabilities read once
-        kname = "cache_scan_kernel"
-    elif dom == "router":
-        flops = 2.0 * w.d * heads * w.N * w.units * args.steps
-        bytes_ = (2.0 * w.d + 4.0 * heads * w.N) * w.units * args.steps   # + scores written
-        kname = f"router_heads_kernel<{w.N},{heads}>"
-    else:
-        flops, bytes_ = algorithmic(w, w.units, heads)
-        flops, bytes_ = flops * args.steps, bytes_ * args.steps
-        kname = f"fused_route_cache_kernel<{w.N},{heads}>"
-    t_flop = flops / (pk["bf16_tflops"] * 1e12)
-    t_byte = bytes_ / (pk["hbm_gbs"] * 1e9)
-    if t_flop >= t_byte:
-        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": pk["bf16_tflops"],
-                "unit": "TFLOP/s", "frac": t_flop / t_s}
-    else:
-        roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
-                "unit": "GB/s", "frac": t_byte / t_s}
-    per_unit, src = committed_traffic(kname, w.name)
-    units_per_launch = w.units * args.steps / max(1, kt[dom]["launches"])
-    roof["traffic"] = None if per_unit is None else per_unit * units_per_launch
-    roof.update({"kernel": kname, "peak_source": f"{pk_src} ({'burst' if roof['bound'] == 'tensor' else 'copy'})",
-                 "avg_launch_ms": avg_ms, "launches": kt[dom]["launches"],
-                 "share_of_step": kt[dom]["ms"] / ms if ms else None})
-    # whole-path roofline (spec definition): max(flops at bf16 peak, bytes at HBM)
-    fl, by = algorithmic(w, w.units, heads)
-    t_roof = max(fl / (pk["bf16_tflops"] * 1e12), by / (pk["hbm_gbs"] * 1e9))
-    path_roof = {"t_roof_ms": 1000 * t_roof, "frac": 1000 * t_roof / ms_per_step,
-                 "bound": "tensor" if fl / (pk["bf16_tflops"] * 1e12) >= by / (pk["hbm_gbs"] * 1e9)
-                 else "hbm"}
-    kernels = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / args.steps}
-               for k, v in kt.items() if v["launches"]}
+    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step)
 
     # end to end through the C ABI from pinned host memory
     e2e = None
     if not args.no_e2e:
-        h_host = torch.empty(hd.shape, dtype=hd.dtype, pin_memory=True)
-        h_host.copy_(hd)
+        held = [hd]                 # the device copy is dropped before the host round trip
         del hd
-        torch.cuda.empty_cache()
-        h_dev = torch.empty(h_host.shape, dtype=h_host.dtype, device=dev)
-        torch.cuda.synchronize()
-
-        def e2e_step():
-            h_dev.copy_(h_host, non_blocking=True)
-            st.init()
-            C.crc_route_and_cache(p, h_dev.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes,
-                                  None, ws.data_ptr(), ws.numel(), stream)
-            return st.read()      # synchronises; reads the step's counters back
-
-        for _ in range(2):
-            e2e_step()
-        if world > 1:
-            dist.barrier()
-        t0 = time.perf_counter()
-        for _ in range(args.steps):
-            r = e2e_step()
-        dt = time.perf_counter() - t0
-        if world > 1:
-            t = torch.tensor([dt], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            dt = float(t.item())
-        assert r["error"] == 0
-        e2e = {"value": units_all * args.steps / dt, "unit": UNIT,
-               "h2d_bytes_per_step": int(h_host.numel() * h_host.element_size()),
-               "d2h_bytes_per_step": int(256 + p.B * p.L * 64),
-               "ms_per_step": 1000 * dt / args.steps}
+        e2e = end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -441,6 +390,184 @@ def main():
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def rooflines(kt, w, heads, steps, ms, ms_per_step):
+    """Roofline of the dominant kernel (timed live over the timed region) and of
+    the whole path (max of flops at bf16 peak and bytes at HBM bandwidth)."""
+    pk, pk_src = peaks()
+    dom = max(("fused", "router", "scan"), key=lambda k: kt[k]["ms"])
+    avg_ms = kt[dom]["ms"] / max(1, kt[dom]["launches"])
+    t_s = kt[dom]["ms"] / 1000.0
+    if dom == "scan":
+        flops = 0.0
+        bytes_ = 4.0 * heads * w.N * w.units * steps          # probabilities read once
+        kname = "cache_scan_kernel"
+    elif dom == "router":
+        flops = 2.0 * w.d * heads * w.N * w.units * steps
+        bytes_ = (2.0 * w.d + 4.0 * heads * w.N) * w.units * steps   # + scores written
+        kname = f"router_heads_kernel<{w.N},{heads}>"
+    else:
+        flops, bytes_ = algorithmic(w, w.units, heads)
+        flops, bytes_ = flops * steps, bytes_ * steps
+        kname = f"fused_route_cache_kernel<{w.N},{heads}>"
+    t_flop = flops / (pk["bf16_tflops"] * 1e12)
+    t_byte = bytes_ / (pk["hbm_gbs"] * 1e9)
+    if t_flop >= t_byte:
+        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": pk["bf16_tflops"],
+                "unit": "TFLOP/s", "frac": t_flop / t_s}
+    else:
+        roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "frac": t_byte / t_s}
+    per_unit, src = committed_traffic(kname, w.name)
+    units_per_launch = w.units * steps / max(1, kt[dom]["launches"])
+    roof["traffic"] = None if per_unit is None else per_unit * units_per_launch
+    roof.update({"kernel": kname, "peak_source": f"{pk_src} ({'burst' if roof['bound'] == 'tensor' else 'copy'})",
+                 "avg_launch_ms": avg_ms, "launches": kt[dom]["launches"],
+                 "share_of_step": kt[dom]["ms"] / ms if ms else None})
+    # whole-path roofline (north-star definition): max(flops at bf16 peak, bytes at HBM)
+    fl, by = algorithmic(w, w.units, heads)
+    t_roof = max(fl / (pk["bf16_tflops"] * 1e12), by / (pk["hbm_gbs"] * 1e9))
+    path_roof = {"t_roof_ms": 1000 * t_roof, "frac": 1000 * t_roof / ms_per_step,
+                 "bound": "tensor" if fl / (pk["bf16_tflops"] * 1e12) >= by / (pk["hbm_gbs"] * 1e9)
+                 else "hbm"}
+    kernels = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / steps}
+               for k, v in kt.items() if v["launches"]}
+    return roof, path_roof, kernels
+
+
+STREAM_BYTES = 128 << 30     # hidden states above this are generated per chunk
+STREAM_CHUNK = 128           # tokens per chunk of a streamed workload
+
+
+def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
+    """Workloads whose hidden states do not fit in HBM (the 1.6 TB large shape).
+    A step walks the T tokens in 128-token chunks: the device generator writes
+    a chunk (untimed; the AR(1) field continues through its carry), and the
+    fused route-and-cache call on it is timed with CUDA events on the stream.
+    The step time is the sum of its timed calls."""
+    import torch
+    import torch.distributed as dist
+    CH = min(STREAM_CHUNK, w.T)
+    n_chunks = (w.T + CH - 1) // CH
+    Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
+    hflat = torch.empty(w.B * CH * w.L * w.d, dtype=torch.bfloat16, device=dev)
+    carry = torch.zeros((w.B, w.L, w.d), dtype=torch.float32, device=dev)
+    ws_bytes = C.crc_fused_workspace_bytes(p)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    st = P.State(p, device=dev)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(n_chunks)]
+
+    def step(timed):
+        st.init()
+        carry.zero_()
+        for c in range(n_chunks):
+            t0 = c * CH
+            n = min(CH, w.T - t0)
+            h = hflat[: w.B * n * w.L * w.d].view(w.B, n, w.L, w.d)
+            P.synth_hidden(w.B, n, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t, rho_l=w.rho_l,
+                           t0=t0, carry=carry, out=h, device=dev)
+            if timed:
+                evs[c][0].record(stream)
+            C.crc_route_and_cache(p, h.data_ptr(), Wd.data_ptr(), n, st.ptr, st.nbytes, None,
+                                  ws.data_ptr(), ws.numel(), stream)
+            if timed:
+                evs[c][1].record(stream)
+        if not timed:
+            return 0.0
+        torch.cuda.synchronize()
+        return sum(a.elapsed_time(b) for a, b in evs)
+
+    for _ in range(max(3, args.warmup)):
+        step(False)
+    stats = st.read()
+    assert stats["error"] == 0 and stats["tokens"] == w.T, stats
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(gpu_id_for_smi(torch, int(os.environ.get("LOCAL_RANK", "0")))) as clk:
+        C.crc_profile_begin()
+        ms = 0.0
+        for _ in range(args.steps):
+            ms += step(True)
+        kt = C.crc_profile_end()
+    stats = st.read()
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_per_step = ms / args.steps
+    units_all = w.units * world
+    value = units_all / (ms_per_step / 1000.0)
+    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step)
+    kernels.pop("synth", None)
+    kernels.pop("state", None)
+    launches = sum(kt[k]["launches"] for k in ("fused", "router", "scan"))
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu, _, _ = cpu_oracle_sample(w, args.cpu_seconds)
+    if rank == 0:
+        m = P.metrics(stats, p)
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": dict(workload_config(w, CH), path="fused, streamed",
+                           workspace_bytes=int(ws_bytes),
+                           timing="sum of per-call CUDA events; chunk generation untimed"),
+            "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
+            "cpu_baseline": cpu,
+            "e2e": None, "e2e_note": "hidden states exceed host and device memory; "
+                                     "generated on the device per chunk",
+            "gpu_launches": int(launches), "clocks": clk.summary(),
+            "policy": {"hit": m["hit"], "adj_hit": m["adj_hit"],
+                       "load_MB_per_token": m["load_per_token_bytes"] / 1e6},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all):
+    """The same metric through the C ABI with the step's inputs copied from
+    pinned host memory and its counters read back, inside the timed region."""
+    import torch
+    import torch.distributed as dist
+    hd = held.pop()
+    h_host = torch.empty(hd.shape, dtype=hd.dtype, pin_memory=True)
+    h_host.copy_(hd)
+    del hd
+    torch.cuda.empty_cache()
+    h_dev = torch.empty(h_host.shape, dtype=h_host.dtype, device=dev)
+    torch.cuda.synchronize()
+
+    def e2e_step():
+        h_dev.copy_(h_host, non_blocking=True)
+        st.init()
+        C.crc_route_and_cache(p, h_dev.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes,
+                              None, ws.data_ptr(), ws.numel(), stream)
+        return st.read()      # synchronises; reads the step's counters back
+
+    for _ in range(2):
+        e2e_step()
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        r = e2e_step()
+    dt = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([dt], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dt = float(t.item())
+    assert r["error"] == 0
+    return {"value": units_all * args.steps / dt, "unit": UNIT,
+            "h2d_bytes_per_step": int(h_host.numel() * h_host.element_size()),
+            "d2h_bytes_per_step": int(256 + p.B * p.L * 64),
+            "ms_per_step": 1000 * dt / args.steps}
 
 
 if __name__ == "__main__":
