@@ -362,49 +362,46 @@ __global__ void __launch_bounds__(512, 1)
 
             // Spatio head: p^S
             if constexpr (H == 3) {
-                float m = -INFINITY, s = 0.f;
+                float m = -INFINITY;
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
 #pragma unroll
-                    for (int i = 0; i < CW; ++i) m = fmaxf(m, z[i]);
+                    m = max_of<CW>(z, m);
                 }
                 // each exp(z - max) is computed once and parked in the
                 // accumulator's own TMEM columns for the normalising pass
+                HeadExp hx;
+                hx.init(m);
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
-#pragma unroll
-                    for (int i = 0; i < CW; ++i) {
-                        z[i] = __expf(z[i] - m);
-                        s += z[i];
-                    }
+                    hx.exp_in_place<CW>(z);
                     tmem_put<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                 }
                 tmem_st_wait();
-                const float r = __frcp_rn(s);
+                const float r = hx.inv();
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
+                    scale_in_place<CW>(z, r);
                     if (ok) {
 #pragma unroll
                         for (int q = 0; q < CW / 4; ++q)
                             pS_p[(size_t)(c * CW / 4 + q) * 128 + row] =
-                                make_float4(__fmul_rn(z[4 * q], r), __fmul_rn(z[4 * q + 1], r),
-                                            __fmul_rn(z[4 * q + 2], r),
-                                            __fmul_rn(z[4 * q + 3], r));
+                                make_float4(z[4 * q], z[4 * q + 1], z[4 * q + 2], z[4 * q + 3]);
                     }
                 }
             }
 
             // native and Temporal heads: s^T and the Top-K set of p^R
-            float mR = -INFINITY, mT = -INFINITY, sR = 0.f, sTs = 0.f;
+            float mR = -INFINITY, mT = -INFINITY;
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
                 tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
@@ -412,12 +409,12 @@ __global__ void __launch_bounds__(512, 1)
                 tmem_ld_wait();
                 pin_cols<CW>(z);
                 pin_cols<CW>(y);
-#pragma unroll
-                for (int i = 0; i < CW; ++i) {
-                    mR = fmaxf(mR, z[i]);
-                    mT = fmaxf(mT, y[i]);
-                }
+                mR = max_of<CW>(z, mR);
+                mT = max_of<CW>(y, mT);
             }
+            HeadExp hR, hT;
+            hR.init(mR);
+            hT.init(mT);
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
                 tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
@@ -425,18 +422,13 @@ __global__ void __launch_bounds__(512, 1)
                 tmem_ld_wait();
                 pin_cols<CW>(z);
                 pin_cols<CW>(y);
-#pragma unroll
-                for (int i = 0; i < CW; ++i) {
-                    z[i] = __expf(z[i] - mR);
-                    y[i] = __expf(y[i] - mT);
-                    sR += z[i];
-                    sTs += y[i];
-                }
+                hR.exp_in_place<CW>(z);
+                hT.exp_in_place<CW>(y);
                 tmem_put<CW>(tbase + (uint32_t)(c * CW), z);
                 tmem_put<CW>(tbase + (uint32_t)(NH + c * CW), y);
             }
             tmem_st_wait();
-            const float rR = __frcp_rn(sR), rT = __frcp_rn(sTs);
+            const float rR = hR.inv(), rT = hT.inv();
             // With a single accumulator, p^R is parked in the spare TMEM columns
             // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
             // before the Top-K selection runs.
@@ -451,13 +443,7 @@ __global__ void __launch_bounds__(512, 1)
                 tmem_ld_wait();
                 pin_cols<CW>(z);
                 pin_cols<CW>(y);
-#pragma unroll
-                for (int i = 0; i < CW; ++i) {
-                    // separately rounded products and sum (no contraction into an
-                    // FMA), exactly as the router writes p^R, p^T and the scan adds them
-                    z[i] = __fmul_rn(z[i], rR);                  // p^R
-                    y[i] = __fadd_rn(z[i], __fmul_rn(y[i], rT));  // s^T
-                }
+                retention_in_place<CW>(z, y, rR, rT);             // z = p^R, y = s^T
                 if (ok) {
 #pragma unroll
                     for (int q = 0; q < CW / 4; ++q)
@@ -503,8 +489,7 @@ __global__ void __launch_bounds__(512, 1)
                         __syncwarp();
                         if (lane == 0) mbar_arrive(&tempty_bar[acc]);
                     }
-#pragma unroll
-                    for (int i = 0; i < CW; ++i) z[i] = __fmul_rn(z[i], rR);   // p^R
+                    scale_in_place<CW>(z, rR);                    // p^R
                 }
 #pragma unroll
                 for (int q = 0; q < CW / 4; ++q) {

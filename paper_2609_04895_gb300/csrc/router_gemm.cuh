@@ -70,21 +70,115 @@ struct RouterArgs {
     int kblocks;         // ceil(d / 64)
 };
 
-// Softmax of one head, in place: exp(z - max z) / sum, fp32.
+// ---------------------------------------------------------------------------
+// Softmax arithmetic, shared by the router and the fused epilogues so that
+// both produce the same bits.  exp(z - m) = 2^(z*log2(e) - m*log2(e)): one
+// FMA per score and the SFU base-2 exponential (approximate, subnormal
+// results flushed to zero).  Scores go in pairs (2j, 2j+1) through packed
+// f32x2 instructions, each lane rounded like its scalar form; the head sum is
+// two partial sums (even and odd positions, in order) added at the end, and
+// p = e * (1 / sum), the reciprocal rounded to nearest.
+// ---------------------------------------------------------------------------
+constexpr float kLog2E = 1.4426950408889634f;
+
+__device__ __forceinline__ uint64_t f2pack(float a, float b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& a, float& b) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2add(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2mul(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ float ex2_sfu(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
+}
+
+// Running maximum over W scores (W even).
+template <int W>
+__device__ __forceinline__ float max_of(const float* z, float m) {
+#pragma unroll
+    for (int i = 0; i < W; i += 2) m = fmax3(m, z[i], z[i + 1]);
+    return m;
+}
+
+// exp(z - m) of a head, in place, chunk after chunk, with its running sum.
+struct HeadExp {
+    uint64_t sum, k, b;
+    __device__ __forceinline__ void init(float m) {
+        const float nb = -__fmul_rn(m, kLog2E);
+        k = f2pack(kLog2E, kLog2E);
+        b = f2pack(nb, nb);
+        sum = f2pack(0.f, 0.f);
+    }
+    template <int W>
+    __device__ __forceinline__ void exp_in_place(float* z) {
+#pragma unroll
+        for (int i = 0; i < W; i += 2) {
+            float u, v;
+            f2unpack(f2fma(f2pack(z[i], z[i + 1]), k, b), u, v);
+            z[i] = ex2_sfu(u);
+            z[i + 1] = ex2_sfu(v);
+            sum = f2add(sum, f2pack(z[i], z[i + 1]));
+        }
+    }
+    __device__ __forceinline__ float inv() const {
+        float u, v;
+        f2unpack(sum, u, v);
+        return __frcp_rn(__fadd_rn(u, v));
+    }
+};
+
+// z <- z * r (probabilities from exps), W even.
+template <int W>
+__device__ __forceinline__ void scale_in_place(float* z, float r) {
+    const uint64_t rr = f2pack(r, r);
+#pragma unroll
+    for (int i = 0; i < W; i += 2) f2unpack(f2mul(f2pack(z[i], z[i + 1]), rr), z[i], z[i + 1]);
+}
+
+// From the native and Temporal exps: z <- p^R = e^R * r^R and
+// y <- s^T = p^R + e^T * r^T, product and sum rounded separately as when the
+// scan adds the stored p^R and p^T.  Scalar on purpose: a packed multiply
+// followed by a packed add may be fused into one packed FMA by the assembler,
+// which rounds once.
+template <int W>
+__device__ __forceinline__ void retention_in_place(float* z, float* y, float rR, float rT) {
+#pragma unroll
+    for (int i = 0; i < W; ++i) {
+        z[i] = __fmul_rn(z[i], rR);
+        y[i] = __fadd_rn(z[i], __fmul_rn(y[i], rT));
+    }
+}
+
+// Softmax of one head held in registers, in place.
 template <int NH>
 __device__ __forceinline__ void head_softmax(float (&z)[NH]) {
-    float m = z[0];
-#pragma unroll
-    for (int i = 1; i < NH; ++i) m = fmaxf(m, z[i]);
-    float s = 0.f;
-#pragma unroll
-    for (int i = 0; i < NH; ++i) {
-        z[i] = __expf(z[i] - m);
-        s += z[i];
-    }
-    const float r = __frcp_rn(s);
-#pragma unroll
-    for (int i = 0; i < NH; ++i) z[i] = __fmul_rn(z[i], r);
+    HeadExp h;
+    h.init(max_of<NH>(z, -INFINITY));
+    h.exp_in_place<NH>(z);
+    scale_in_place<NH>(z, h.inv());
 }
 
 template <int NH, int H>
