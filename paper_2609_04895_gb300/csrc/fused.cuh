@@ -590,18 +590,21 @@ __global__ void __launch_bounds__(512, 1)
             const int steps = imin(a.TB, a.T - tb * a.TB);
             const int last_row = sbi * a.TB + steps - 1;
             // inputs of step tbi: s^T, the Top-K bits and p^S of the predecessor
-            auto fetch = [&](int tbi, float (&sT)[V], float (&pS)[V], uint32_t& sel) {
+            // the first step of this block with a causal predecessor (refinement)
+            const int refine_from =
+                (int)(t0g + (int64_t)tb * a.TB >= 1 ? 0 : 1 - (t0g + (int64_t)tb * a.TB));
+            // the Top-K word is fetched whole and its bits taken at use, so the
+            // load stays in flight across the step instead of stalling the fetch
+            auto fetch = [&](int tbi, float (&sT)[V], float (&pS)[V], uint32_t& selw) {
                 const int r = sbi * a.TB + tbi;
 #pragma unroll
                 for (int v = 0; v < V; ++v) sT[v] = pS[v] = 0.f;
-                sel = 0u;
+                selw = 0u;
                 if (!has) return;
                 ring_vec<V>(own + RL::ST, lane, r, sT);
-                sel = (__ldcg(reinterpret_cast<const uint32_t*>(own + RL::SEL) +
-                              (size_t)(e0 >> 5) * 128 + r) >>
-                       (e0 & 31)) &
-                      ((1u << V) - 1u);
-                if (want_s && (t0g + tb * a.TB + tbi >= 1)) {
+                selw = __ldcg(reinterpret_cast<const uint32_t*>(own + RL::SEL) +
+                              (size_t)(e0 >> 5) * 128 + r);
+                if (want_s && tbi >= refine_from) {
                     if (l > 0) {
                         ring_vec<V>(psl + RL::PS, lane, r, pS);
                     } else if (tbi > 0) {
@@ -640,10 +643,10 @@ __global__ void __launch_bounds__(512, 1)
                 uint32_t nsel = 0u;
                 if (tbi + 1 < steps) fetch(tbi + 1, nT, nS, nsel);
                 if ((tbi & 7) == 0) prefetch_rows(tbi + 24);
-                const bool refine = want_s && (t0g + tb * a.TB + tbi >= 1);
+                const bool refine = want_s && tbi >= refine_from;
                 int nD;
-                scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R, csel,
-                                         &nD);
+                scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R,
+                                         (csel >> (e0 & 31)) & ((1u << V) - 1u), &nD);
 #pragma unroll
                 for (int v = 0; v < V; ++v) {
                     cT[v] = nT[v];
