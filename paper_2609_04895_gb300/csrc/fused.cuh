@@ -161,6 +161,180 @@ __device__ __forceinline__ void ring_vec(const uint8_t* base, int lane, int r, f
     }
 }
 
+// The scan role of the fused kernels (one warp per item): items (chain,
+// block of TB tokens) come from a global counter in token order; each waits
+// (bounded) for the chain's previous block and for the tiles it reads (a tile
+// is complete when `publishers` epilogue warps have published it), runs
+// Algorithm 2 / 1 on each token (scan_apply) and releases the tiles through
+// the monotonic reader counters.
+template <int NH, int V, bool ALL_VALID>
+__device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* err,
+                                                uint32_t* abort_flag, int64_t t0g,
+                                                uint32_t parity, int lane, uint32_t publishers) {
+    using RL = RingLayout<NH>;
+    StateLayout lay = state_layout(a.B, a.L, a.N);
+    ChainState* chains = reinterpret_cast<ChainState*>(a.state + lay.chains);
+    float* retention = reinterpret_cast<float*>(a.state + lay.retention);
+    float* carry = reinterpret_cast<float*>(a.state + lay.carry);
+    const int N = a.N, L = a.L;
+    uint32_t valid = 0u;
+#pragma unroll
+    for (int v = 0; v < V; ++v)
+        if (lane * V + v < N) valid |= 1u << v;
+    const bool has = valid != 0u;
+    const bool want_s = a.R > 0;
+    const uint32_t e0 = (uint32_t)lane * V;
+    while (true) {
+        uint32_t item = 0u;
+        if (lane == 0) item = atomicAdd(&a.ctl[0], 1u);
+        item = __shfl_sync(kFull, item, 0);
+        if (item >= (uint32_t)a.n_items) break;
+        const int tb = (int)(item / (uint32_t)(L * a.B));
+        const int rem = (int)(item % (uint32_t)(L * a.B));
+        const int l = rem / a.B, b = rem % a.B;
+        const int bg = b / a.SB, sbi = b % a.SB;
+        const int chain = b * L + l;
+        const int k_own = (tb * L + l) * a.n_bg + bg;
+        const int k_ps = (tb * L + (l > 0 ? l - 1 : L - 1)) * a.n_bg + bg;
+        const int k_prev = (l == 0 && tb > 0) ? ((tb - 1) * L + L - 1) * a.n_bg + bg : -1;
+        const bool read_ps = want_s && (l > 0 || a.TB >= 2);
+        // wait for the chain's previous block and the tiles this item reads
+        bool ok = true;
+        if (lane == 0) {
+            ok = wait_geq(&a.prog[chain], (uint32_t)tb, abort_flag, err);
+            auto ready = [&](int k) {
+                return wait_geq(&a.tile_done[k % a.ring], publishers * (uint32_t)(k / a.ring + 1),
+                                abort_flag, err);
+            };
+            ok = ok && ready(k_own);
+            if (read_ps) ok = ok && ready(k_ps);
+            if (want_s && k_prev >= 0) ok = ok && ready(k_prev);
+        }
+        ok = __shfl_sync(kFull, ok, 0);
+        if (!ok) break;
+
+        ChainState& cs = chains[chain];
+        ChainRegs<V> cr;
+        cr.cache = lane_bits_cg<V>(cs.bits, lane, N);
+        cr.count = (int)__reduce_add_sync(kFull, (uint32_t)__popc(cr.cache));
+        {
+            Vec<V> x = ldcg_vec<V>(retention + (size_t)chain * N + e0, has);
+#pragma unroll
+            for (int v = 0; v < V; ++v) cr.aT[v] = x.v[v];
+        }
+        cr.hits = cr.misses = cr.pro = 0u;
+        const uint8_t* own = a.ring_base + (size_t)(k_own % a.ring) * a.slot_bytes;
+        const uint8_t* psl = a.ring_base + (size_t)(k_ps % a.ring) * a.slot_bytes;
+        const uint8_t* prv =
+            k_prev >= 0 ? a.ring_base + (size_t)(k_prev % a.ring) * a.slot_bytes : nullptr;
+        const float* carry_in = carry + ((size_t)parity * a.B + b) * N + e0;
+        const int steps = imin(a.TB, a.T - tb * a.TB);
+        const int last_row = sbi * a.TB + steps - 1;
+        // inputs of step tbi: s^T, the Top-K bits and p^S of the predecessor
+        // the first step of this block with a causal predecessor (refinement)
+        const int refine_from =
+            (int)(t0g + (int64_t)tb * a.TB >= 1 ? 0 : 1 - (t0g + (int64_t)tb * a.TB));
+        // the Top-K word is fetched whole and its bits taken at use, so the
+        // load stays in flight across the step instead of stalling the fetch
+        auto fetch = [&](int tbi, float (&sT)[V], float (&pS)[V], uint32_t& selw) {
+            const int r = sbi * a.TB + tbi;
+#pragma unroll
+            for (int v = 0; v < V; ++v) sT[v] = pS[v] = 0.f;
+            selw = 0u;
+            if (!has) return;
+            ring_vec<V>(own + RL::ST, lane, r, sT);
+            selw = __ldcg(reinterpret_cast<const uint32_t*>(own + RL::SEL) +
+                          (size_t)(e0 >> 5) * 128 + r);
+            if (want_s && tbi >= refine_from) {
+                if (l > 0) {
+                    ring_vec<V>(psl + RL::PS, lane, r, pS);
+                } else if (tbi > 0) {
+                    ring_vec<V>(psl + RL::PS, lane, r - 1, pS);
+                } else if (prv) {
+                    ring_vec<V>(prv + RL::PS, lane, sbi * a.TB + a.TB - 1, pS);
+                } else {
+                    Vec<V> x = ldcg_vec<V>(carry_in, true);
+#pragma unroll
+                    for (int v = 0; v < V; ++v) pS[v] = x.v[v];
+                }
+            }
+        };
+        // Pull the next 128-byte lines of this lane's chunks into L2 ahead of
+        // use (rows r .. r+7 of a chunk share one line; sel words 32 rows).
+        auto prefetch_rows = [&](int tbi) {
+            if (!has || tbi >= steps) return;
+            const int r = sbi * a.TB + tbi;
+            const int ch = (int)(e0 >> 2);
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(own + RL::ST +
+                                                           ((size_t)ch * 128 + r) * 16));
+            if (want_s)
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(psl + RL::PS +
+                                                               ((size_t)ch * 128 + r) * 16));
+            if ((tbi & 31) == 0)
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(
+                    own + RL::SEL + ((size_t)(e0 >> 5) * 128 + r) * 4));
+        };
+        prefetch_rows(8);
+        prefetch_rows(16);
+        float cT[V], cS[V];
+        uint32_t csel;
+        fetch(0, cT, cS, csel);
+        for (int tbi = 0; tbi < steps; ++tbi) {
+            float nT[V], nS[V];
+            uint32_t nsel = 0u;
+            if (tbi + 1 < steps) fetch(tbi + 1, nT, nS, nsel);
+            if ((tbi & 7) == 0) prefetch_rows(tbi + 24);
+            const bool refine = want_s && tbi >= refine_from;
+            int nD;
+            scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R,
+                                     (csel >> (e0 & 31)) & ((1u << V) - 1u), &nD);
+#pragma unroll
+            for (int v = 0; v < V; ++v) {
+                cT[v] = nT[v];
+                cS[v] = nS[v];
+            }
+            csel = nsel;
+        }
+        // the last layer hands p^S of the call's last token to layer 0 of the next call
+        if (l == L - 1 && want_s && tb * a.TB + a.TB >= a.T && steps > 0 && has) {
+            float pl[V];
+            ring_vec<V>(own + RL::PS, lane, last_row, pl);   // has: lane owns experts
+            float* dst = carry + ((size_t)(parity ^ 1u) * a.B + b) * N + e0;
+#pragma unroll
+            for (int v = 0; v < V; ++v)
+                if (lane * V + v < N) dst[v] = pl[v];
+        }
+        // store the chain
+        const int NW = (N + 31) >> 5;
+        for (int w = 0; w < NW; ++w) {
+            const uint32_t contrib = (has && (e0 >> 5) == (uint32_t)w) ? (cr.cache << (e0 & 31)) : 0u;
+            const uint32_t wd = __reduce_or_sync(kFull, contrib);
+            if (lane == 0) cs.bits[w] = wd;
+        }
+        if (has) {
+#pragma unroll
+            for (int v = 0; v < V; ++v)
+                if (lane * V + v < N) retention[(size_t)chain * N + e0 + v] = cr.aT[v];
+        }
+        if (lane == 0) {
+            cs.hits = __ldcg(&cs.hits) + cr.hits;
+            cs.misses = __ldcg(&cs.misses) + cr.misses;
+            cs.proactive = __ldcg(&cs.proactive) + cr.pro;
+        }
+        // release the tiles and the chain
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) {
+            atomicAdd(&a.readers[k_own % a.ring], 1u);
+            if (want_s) {
+                if (l > 0 || a.TB >= 2) atomicAdd(&a.readers[k_ps % a.ring], 1u);
+                if (k_prev >= 0) atomicAdd(&a.readers[k_prev % a.ring], 1u);
+            }
+            atomicExch(&a.prog[chain], (uint32_t)(tb + 1));
+        }
+    }
+}
+
 template <int NH, int H>
 struct FusedCfg {
     using RC = RouterCfg<NH, H>;
@@ -183,6 +357,18 @@ __global__ void __launch_bounds__(512, 1)
     using RL = RingLayout<NH>;
     constexpr int CW = Cfg::CW;
     constexpr int NCHK = Cfg::NCHK;
+    // exps of chunk c in place, into the accumulator of the head half it covers
+    auto chunk_exp = [](int c, float* v, HeadExp& e0, HeadExp& e1) {
+        if constexpr (NCHK >= 2) {
+            if (c < NCHK / 2)
+                e0.exp_in_place<CW>(v);
+            else
+                e1.exp_in_place<CW>(v);
+        } else {                                        // one chunk holds both halves
+            e0.exp_in_place<CW / 2>(v);
+            e1.exp_in_place<CW / 2>(v + CW / 2);
+        }
+    };
 
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -373,18 +559,19 @@ __global__ void __launch_bounds__(512, 1)
                 }
                 // each exp(z - max) is computed once and parked in the
                 // accumulator's own TMEM columns for the normalising pass
-                HeadExp hx;
-                hx.init(m);
+                HeadExp x0, x1;
+                x0.init(m);
+                x1.init(m);
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
-                    hx.exp_in_place<CW>(z);
+                    chunk_exp(c, z, x0, x1);
                     tmem_put<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                 }
                 tmem_st_wait();
-                const float r = hx.inv();
+                const float r = head_inv(x0.part(), x1.part());
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
@@ -412,9 +599,11 @@ __global__ void __launch_bounds__(512, 1)
                 mR = max_of<CW>(z, mR);
                 mT = max_of<CW>(y, mT);
             }
-            HeadExp hR, hT;
-            hR.init(mR);
-            hT.init(mT);
+            HeadExp r0, r1, t0, t1;
+            r0.init(mR);
+            r1.init(mR);
+            t0.init(mT);
+            t1.init(mT);
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
                 tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
@@ -422,13 +611,13 @@ __global__ void __launch_bounds__(512, 1)
                 tmem_ld_wait();
                 pin_cols<CW>(z);
                 pin_cols<CW>(y);
-                hR.exp_in_place<CW>(z);
-                hT.exp_in_place<CW>(y);
+                chunk_exp(c, z, r0, r1);
+                chunk_exp(c, y, t0, t1);
                 tmem_put<CW>(tbase + (uint32_t)(c * CW), z);
                 tmem_put<CW>(tbase + (uint32_t)(NH + c * CW), y);
             }
             tmem_st_wait();
-            const float rR = hR.inv(), rT = hT.inv();
+            const float rR = head_inv(r0.part(), r1.part()), rT = head_inv(t0.part(), t1.part());
             // With a single accumulator, p^R is parked in the spare TMEM columns
             // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
             // before the Top-K selection runs.
@@ -530,170 +719,8 @@ __global__ void __launch_bounds__(512, 1)
             if (!ok) break;
         }
     } else if (hdr_ok) {
-        // ------------------------------------------------------------ scan
-        StateLayout lay = state_layout(a.B, a.L, a.N);
-        ChainState* chains = reinterpret_cast<ChainState*>(a.state + lay.chains);
-        float* retention = reinterpret_cast<float*>(a.state + lay.retention);
-        float* carry = reinterpret_cast<float*>(a.state + lay.carry);
-        const int N = a.N, L = a.L;
-        uint32_t valid = 0u;
-#pragma unroll
-        for (int v = 0; v < V; ++v)
-            if (lane * V + v < N) valid |= 1u << v;
-        const bool has = valid != 0u;
-        const bool want_s = a.R > 0;
-        const uint32_t e0 = (uint32_t)lane * V;
-        while (true) {
-            uint32_t item = 0u;
-            if (lane == 0) item = atomicAdd(&a.ctl[0], 1u);
-            item = __shfl_sync(kFull, item, 0);
-            if (item >= (uint32_t)a.n_items) break;
-            const int tb = (int)(item / (uint32_t)(L * a.B));
-            const int rem = (int)(item % (uint32_t)(L * a.B));
-            const int l = rem / a.B, b = rem % a.B;
-            const int bg = b / a.SB, sbi = b % a.SB;
-            const int chain = b * L + l;
-            const int k_own = (tb * L + l) * a.n_bg + bg;
-            const int k_ps = (tb * L + (l > 0 ? l - 1 : L - 1)) * a.n_bg + bg;
-            const int k_prev = (l == 0 && tb > 0) ? ((tb - 1) * L + L - 1) * a.n_bg + bg : -1;
-            const bool read_ps = want_s && (l > 0 || a.TB >= 2);
-            // wait for the chain's previous block and the tiles this item reads
-            bool ok = true;
-            if (lane == 0) {
-                ok = wait_geq(&a.prog[chain], (uint32_t)tb, abort_flag, err);
-                auto ready = [&](int k) {
-                    return wait_geq(&a.tile_done[k % a.ring], 4u * (uint32_t)(k / a.ring + 1),
-                                    abort_flag, err);
-                };
-                ok = ok && ready(k_own);
-                if (read_ps) ok = ok && ready(k_ps);
-                if (want_s && k_prev >= 0) ok = ok && ready(k_prev);
-            }
-            ok = __shfl_sync(kFull, ok, 0);
-            if (!ok) break;
-
-            ChainState& cs = chains[chain];
-            ChainRegs<V> cr;
-            cr.cache = lane_bits_cg<V>(cs.bits, lane, N);
-            cr.count = (int)__reduce_add_sync(kFull, (uint32_t)__popc(cr.cache));
-            {
-                Vec<V> x = ldcg_vec<V>(retention + (size_t)chain * N + e0, has);
-#pragma unroll
-                for (int v = 0; v < V; ++v) cr.aT[v] = x.v[v];
-            }
-            cr.hits = cr.misses = cr.pro = 0u;
-            const uint8_t* own = a.ring_base + (size_t)(k_own % a.ring) * a.slot_bytes;
-            const uint8_t* psl = a.ring_base + (size_t)(k_ps % a.ring) * a.slot_bytes;
-            const uint8_t* prv =
-                k_prev >= 0 ? a.ring_base + (size_t)(k_prev % a.ring) * a.slot_bytes : nullptr;
-            const float* carry_in = carry + ((size_t)parity * a.B + b) * N + e0;
-            const int steps = imin(a.TB, a.T - tb * a.TB);
-            const int last_row = sbi * a.TB + steps - 1;
-            // inputs of step tbi: s^T, the Top-K bits and p^S of the predecessor
-            // the first step of this block with a causal predecessor (refinement)
-            const int refine_from =
-                (int)(t0g + (int64_t)tb * a.TB >= 1 ? 0 : 1 - (t0g + (int64_t)tb * a.TB));
-            // the Top-K word is fetched whole and its bits taken at use, so the
-            // load stays in flight across the step instead of stalling the fetch
-            auto fetch = [&](int tbi, float (&sT)[V], float (&pS)[V], uint32_t& selw) {
-                const int r = sbi * a.TB + tbi;
-#pragma unroll
-                for (int v = 0; v < V; ++v) sT[v] = pS[v] = 0.f;
-                selw = 0u;
-                if (!has) return;
-                ring_vec<V>(own + RL::ST, lane, r, sT);
-                selw = __ldcg(reinterpret_cast<const uint32_t*>(own + RL::SEL) +
-                              (size_t)(e0 >> 5) * 128 + r);
-                if (want_s && tbi >= refine_from) {
-                    if (l > 0) {
-                        ring_vec<V>(psl + RL::PS, lane, r, pS);
-                    } else if (tbi > 0) {
-                        ring_vec<V>(psl + RL::PS, lane, r - 1, pS);
-                    } else if (prv) {
-                        ring_vec<V>(prv + RL::PS, lane, sbi * a.TB + a.TB - 1, pS);
-                    } else {
-                        Vec<V> x = ldcg_vec<V>(carry_in, true);
-#pragma unroll
-                        for (int v = 0; v < V; ++v) pS[v] = x.v[v];
-                    }
-                }
-            };
-            // Pull the next 128-byte lines of this lane's chunks into L2 ahead of
-            // use (rows r .. r+7 of a chunk share one line; sel words 32 rows).
-            auto prefetch_rows = [&](int tbi) {
-                if (!has || tbi >= steps) return;
-                const int r = sbi * a.TB + tbi;
-                const int ch = (int)(e0 >> 2);
-                asm volatile("prefetch.global.L2 [%0];" ::"l"(own + RL::ST +
-                                                               ((size_t)ch * 128 + r) * 16));
-                if (want_s)
-                    asm volatile("prefetch.global.L2 [%0];" ::"l"(psl + RL::PS +
-                                                                   ((size_t)ch * 128 + r) * 16));
-                if ((tbi & 31) == 0)
-                    asm volatile("prefetch.global.L2 [%0];" ::"l"(
-                        own + RL::SEL + ((size_t)(e0 >> 5) * 128 + r) * 4));
-            };
-            prefetch_rows(8);
-            prefetch_rows(16);
-            float cT[V], cS[V];
-            uint32_t csel;
-            fetch(0, cT, cS, csel);
-            for (int tbi = 0; tbi < steps; ++tbi) {
-                float nT[V], nS[V];
-                uint32_t nsel = 0u;
-                if (tbi + 1 < steps) fetch(tbi + 1, nT, nS, nsel);
-                if ((tbi & 7) == 0) prefetch_rows(tbi + 24);
-                const bool refine = want_s && tbi >= refine_from;
-                int nD;
-                scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R,
-                                         (csel >> (e0 & 31)) & ((1u << V) - 1u), &nD);
-#pragma unroll
-                for (int v = 0; v < V; ++v) {
-                    cT[v] = nT[v];
-                    cS[v] = nS[v];
-                }
-                csel = nsel;
-            }
-            // the last layer hands p^S of the call's last token to layer 0 of the next call
-            if (l == L - 1 && want_s && tb * a.TB + a.TB >= a.T && steps > 0 && has) {
-                float pl[V];
-                ring_vec<V>(own + RL::PS, lane, last_row, pl);   // has: lane owns experts
-                float* dst = carry + ((size_t)(parity ^ 1u) * a.B + b) * N + e0;
-#pragma unroll
-                for (int v = 0; v < V; ++v)
-                    if (lane * V + v < N) dst[v] = pl[v];
-            }
-            // store the chain
-            const int NW = (N + 31) >> 5;
-            for (int w = 0; w < NW; ++w) {
-                const uint32_t contrib = (has && (e0 >> 5) == (uint32_t)w) ? (cr.cache << (e0 & 31)) : 0u;
-                const uint32_t wd = __reduce_or_sync(kFull, contrib);
-                if (lane == 0) cs.bits[w] = wd;
-            }
-            if (has) {
-#pragma unroll
-                for (int v = 0; v < V; ++v)
-                    if (lane * V + v < N) retention[(size_t)chain * N + e0 + v] = cr.aT[v];
-            }
-            if (lane == 0) {
-                cs.hits = __ldcg(&cs.hits) + cr.hits;
-                cs.misses = __ldcg(&cs.misses) + cr.misses;
-                cs.proactive = __ldcg(&cs.proactive) + cr.pro;
-            }
-            // release the tiles and the chain
-            __threadfence();
-            __syncwarp();
-            if (lane == 0) {
-                atomicAdd(&a.readers[k_own % a.ring], 1u);
-                if (want_s) {
-                    if (l > 0 || a.TB >= 2) atomicAdd(&a.readers[k_ps % a.ring], 1u);
-                    if (k_prev >= 0) atomicAdd(&a.readers[k_prev % a.ring], 1u);
-                }
-                atomicExch(&a.prog[chain], (uint32_t)(tb + 1));
-            }
-        }
+        fused_scan_role<NH, V, ALL_VALID>(a, err, abort_flag, t0g, parity, lane, 4u);
     }
-
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {

@@ -75,9 +75,11 @@ struct RouterArgs {
 // both produce the same bits.  exp(z - m) = 2^(z*log2(e) - m*log2(e)): one
 // FMA per score and the SFU base-2 exponential (approximate, subnormal
 // results flushed to zero).  Scores go in pairs (2j, 2j+1) through packed
-// f32x2 instructions, each lane rounded like its scalar form; the head sum is
-// two partial sums (even and odd positions, in order) added at the end, and
-// p = e * (1 / sum), the reciprocal rounded to nearest.
+// f32x2 instructions, each lane rounded like its scalar form.  The head sum
+// is (sum over the first half of the experts) + (sum over the second half),
+// each half's sum the total of two running partial sums (even and odd
+// positions, in order); then p = e * (1 / sum), the reciprocal rounded to
+// nearest.  (Halves let two CTAs that hold one half each agree on the sum.)
 // ---------------------------------------------------------------------------
 constexpr float kLog2E = 1.4426950408889634f;
 
@@ -143,12 +145,16 @@ struct HeadExp {
             sum = f2add(sum, f2pack(z[i], z[i + 1]));
         }
     }
-    __device__ __forceinline__ float inv() const {
+    // this accumulator's sum (one half of a head)
+    __device__ __forceinline__ float part() const {
         float u, v;
         f2unpack(sum, u, v);
-        return __frcp_rn(__fadd_rn(u, v));
+        return __fadd_rn(u, v);
     }
 };
+
+// 1 / (first-half sum + second-half sum): a head's normaliser.
+__device__ __forceinline__ float head_inv(float s0, float s1) { return __frcp_rn(__fadd_rn(s0, s1)); }
 
 // z <- z * r (probabilities from exps), W even.
 template <int W>
@@ -175,10 +181,13 @@ __device__ __forceinline__ void retention_in_place(float* z, float* y, float rR,
 // Softmax of one head held in registers, in place.
 template <int NH>
 __device__ __forceinline__ void head_softmax(float (&z)[NH]) {
-    HeadExp h;
-    h.init(max_of<NH>(z, -INFINITY));
-    h.exp_in_place<NH>(z);
-    scale_in_place<NH>(z, h.inv());
+    const float m = max_of<NH>(z, -INFINITY);
+    HeadExp h0, h1;
+    h0.init(m);
+    h1.init(m);
+    h0.exp_in_place<NH / 2>(z);
+    h1.exp_in_place<NH / 2>(z + NH / 2);
+    scale_in_place<NH>(z, head_inv(h0.part(), h1.part()));
 }
 
 template <int NH, int H>
