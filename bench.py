@@ -216,6 +216,16 @@ def cpu_oracle_sample(w, seconds: float):
                       f"(fp64 router heads + literal scan), {dt:.1f} s wall"}, units, dt
 
 
+def policy_report(P, stats, p, m):
+    """Hit, AdjHit, Load/token (Sec. 4.1) and the overlap model's exposed
+    loading cost per decode token at no and at full prefetch overlap, in
+    expert transfers (multiply by the seconds per expert transfer)."""
+    return {"hit": m["hit"], "adj_hit": m["adj_hit"],
+            "load_MB_per_token": m["load_per_token_bytes"] / 1e6,
+            "t_load_transfers_per_token": {"eta0": P.load_time(stats, p, 1.0, 0.0),
+                                           "eta1": P.load_time(stats, p, 1.0, 1.0)}}
+
+
 def workload_of(args):
     w = S.WORKLOADS[args.workload]
     if args.tokens:
@@ -383,8 +393,7 @@ def main():
             "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
             "clocks": clk.summary(),
-            "policy": {"hit": m["hit"], "adj_hit": m["adj_hit"],
-                       "load_MB_per_token": m["load_per_token_bytes"] / 1e6},
+            "policy": policy_report(P, stats, p, m),
         }
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -522,8 +531,7 @@ def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
             "e2e": None, "e2e_note": "hidden states exceed host and device memory; "
                                      "generated on the device per chunk",
             "gpu_launches": int(launches), "clocks": clk.summary(),
-            "policy": {"hit": m["hit"], "adj_hit": m["adj_hit"],
-                       "load_MB_per_token": m["load_per_token_bytes"] / 1e6},
+            "policy": policy_report(P, stats, p, m),
         }
         print(json.dumps(line), flush=True)
     if world > 1:

@@ -197,6 +197,15 @@ def metrics(A: float, D: float, P: float, T: float, s_exp_bytes: float) -> dict:
     return {"hit": h.value, "adj_hit": a.value, "load_per_token": ld.value}
 
 
+def load_time(D: float, P: float, T: float, c_exp: float, eta: float) -> float:
+    """Modeled exposed expert-loading cost per decode token (appendix on
+    asynchronous transfer overlap): c_exp / T * (D + (1 - eta) * P)."""
+    f = lib().oracle_load_time
+    f.restype = ctypes.c_double
+    f.argtypes = [ctypes.c_double] * 5
+    return f(float(D), float(P), float(T), float(c_exp), float(eta))
+
+
 def run(hidden_bits: np.ndarray, w_bits: np.ndarray, N: int, K: int, C: int, R: int,
         margins: bool = True, nthreads: int | None = None) -> dict:
     """End-to-end fp64 oracle: router probabilities then the scan."""

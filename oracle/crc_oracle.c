@@ -164,6 +164,15 @@ static double rel_gap(double a, double b)
 /* ------------------------------------------------------------------------ */
 /* reporting (Sec. 4.1 Metrics)                                              */
 /* ------------------------------------------------------------------------ */
+/* Exposed expert-loading cost per decode token under the overlap model of the
+ * appendix on asynchronous transfer overlap: demand transfers fully exposed, a
+ * fraction eta of proactive transfer time hidden, c_exp seconds per expert:
+ * t_load(eta) = c_exp / T * (D + (1 - eta) * P). */
+double oracle_load_time(double D, double P, double T, double c_exp, double eta)
+{
+    return c_exp / T * (D + (1.0 - eta) * P);
+}
+
 /* Hit = 1 - D/A, AdjHit = (A - D)/(A + P), Load/token = (D + P) * S_exp / T. */
 void oracle_metrics(double A, double D, double P, double T, double s_exp,
                     double *hit, double *adj_hit, double *load_per_token)

@@ -329,6 +329,20 @@ def synth_hidden(B, T, L, d, seed=0, rho_t=0.9, rho_l=0.8, t0=0, carry=None, att
     return out, carry
 
 
+def load_time(stats: dict, p: crc_problem, c_exp: float, eta: float) -> float:
+    """Exposed expert-loading cost per decode token under the paper's overlap
+    model (appendix on asynchronous transfer overlap): every expert transfer
+    takes c_exp seconds, demand transfers are fully exposed and a fraction eta
+    of the proactive ones is hidden by computation:
+    t_load(eta) = c_exp / T * (D + (1 - eta) * P), T = decode tokens."""
+    if not 0.0 <= eta <= 1.0:
+        raise ValueError("eta must lie in [0, 1]")
+    tokens = stats["tokens"] * p.B
+    if tokens == 0:
+        return 0.0
+    return c_exp / tokens * (stats["misses"] + (1.0 - eta) * stats["proactive"])
+
+
 def metrics(stats: dict, p: crc_problem) -> dict:
     """Hit, AdjHit and Load/token (bytes per decode token) of Sec. 4.1 from
     the totals of crc_state_read; decode tokens = streams x tokens per stream."""

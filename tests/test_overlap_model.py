@@ -1,0 +1,79 @@
+"""The exposed-loading model of the appendix on asynchronous transfer overlap:
+t_load(eta) = c_exp / T * (D + (1 - eta) * P).
+
+Pinned to the two endpoint identities the paper states in terms of its
+reported metrics, t_load(1) = A c_exp / T * (1 - Hit) and
+t_load(0) = (A + P) c_exp / T * (1 - AdjHit) (Hit and AdjHit as in Sec. 4.1),
+to the bounds D c_exp / T <= t_load <= (D + P) c_exp / T, to linearity in eta,
+and to the printed Table 1-3 cells through the Load identity; the product's
+host-side function agrees with the oracle's.
+"""
+import os
+
+import numpy as np
+import pytest
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def test_endpoints_match_the_hit_identities(oracle_lib):
+    rng = np.random.default_rng(5)
+    for _ in range(200):
+        A = float(rng.integers(1, 10_000))
+        D = float(rng.integers(0, int(A) + 1))
+        P = float(rng.integers(0, 5_000))
+        T = float(rng.integers(1, 1_000))
+        c = float(rng.uniform(1e-5, 1e-2))
+        m = oracle_lib.metrics(A, D, P, T, 1.0)
+        assert oracle_lib.load_time(D, P, T, c, 1.0) == pytest.approx(A * c / T * (1 - m["hit"]),
+                                                                     rel=1e-12, abs=1e-18)
+        assert oracle_lib.load_time(D, P, T, c, 0.0) == pytest.approx(
+            (A + P) * c / T * (1 - m["adj_hit"]), rel=1e-12, abs=1e-18)
+
+
+def test_bounds_and_linearity(oracle_lib):
+    rng = np.random.default_rng(6)
+    for _ in range(100):
+        D, P = float(rng.integers(0, 1000)), float(rng.integers(0, 1000))
+        T, c = float(rng.integers(1, 50)), float(rng.uniform(0.1, 2.0))
+        lo, hi = D * c / T, (D + P) * c / T
+        ts = [oracle_lib.load_time(D, P, T, c, e) for e in np.linspace(0, 1, 11)]
+        assert all(lo - 1e-12 <= t <= hi + 1e-12 for t in ts)
+        assert all(a >= b for a, b in zip(ts, ts[1:]))          # more overlap, less exposed cost
+        assert ts[5] == pytest.approx(0.5 * (ts[0] + ts[10]), rel=1e-12)
+    assert oracle_lib.load_time(7, 0, 3, 1, 0.3) == oracle_lib.load_time(7, 0, 3, 1, 0.9)  # P = 0
+
+
+def test_printed_cells_through_the_load_identity(oracle_lib):
+    # per decode token: A = L*K accesses; D = (1 - Hit) A; D + P = Load / S_exp
+    model = {"qwen3": (48, 8, 3 * 2048 * 768 * 2), "gptoss": (24, 4, 3 * 2880 * 2880 * 2)}
+    n = 0
+    with open(os.path.join(HERE, "golden", "paper_metrics.txt")) as f:
+        for line in f:
+            if not line.strip() or line.startswith("#"):
+                continue
+            src, m, meth, task, hit, adj, load = line.split()
+            if adj == "-":
+                continue
+            L, K, s_exp = model[m]
+            A = float(L * K)
+            D = (1 - float(hit) / 100) * A
+            P = float(load) * 1e6 / s_exp - D
+            c = 1.0
+            # fully hidden prefetch leaves the demand misses; none hidden, every transfer
+            assert oracle_lib.load_time(D, P, 1.0, c, 1.0) == pytest.approx(D, rel=1e-12)
+            assert oracle_lib.load_time(D, P, 1.0, c, 0.0) * s_exp / 1e6 == pytest.approx(
+                float(load), rel=1e-9)
+            n += 1
+    assert n > 0
+
+
+def test_product_function_matches_the_oracle(oracle_lib):
+    from paper_2609_04895_gb300 import crc
+    p = crc.problem(L=4, N=16, K=2, d=256, C=4, R=1, B=3, expert_bytes=1 << 20)
+    stats = {"misses": 37, "proactive": 11, "tokens": 25, "accesses": 4 * 25 * 2 * 3}
+    for eta in (0.0, 0.3, 1.0):
+        assert crc.load_time(stats, p, 2e-3, eta) == pytest.approx(
+            oracle_lib.load_time(37, 11, 25 * 3, 2e-3, eta), rel=1e-15)
+    with pytest.raises(ValueError):
+        crc.load_time(stats, p, 1.0, 1.5)
