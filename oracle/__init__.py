@@ -148,6 +148,37 @@ def scan(probs: np.ndarray, K: int, C: int, R: int, trace: bool = True,
     return res
 
 
+# comparison policies (numbering shared with nothing: the oracle's own)
+POLICIES = {"lru": 1, "lfu": 2, "lrfu": 3, "spatio_lru": 4}
+
+
+def policy_scan(probs: np.ndarray, K: int, C: int, R: int, policy: str, lambda2: int = 1,
+                trace: bool = True) -> dict:
+    """Cache scan under a comparison policy (LRU, LFU, LRFU with
+    lambda = lambda2 / 2, Spatio-only with LRU demand eviction) over fp32
+    probabilities [B][T][L][3][N]; see the readings in crc_oracle.c."""
+    p = np.ascontiguousarray(probs, dtype=np.float32)
+    B, T, L, three, N = p.shape
+    assert three == 3
+    NW = (N + 31) // 32
+    res = {
+        "topk": np.zeros((B, T, L, K), np.uint8) if trace else None,
+        "misses": np.zeros((B, T, L), np.uint8) if trace else None,
+        "proactive": np.zeros((B, T, L), np.uint8) if trace else None,
+        "cache_bits": np.zeros((B, L, NW), np.uint32),
+        "aux": np.zeros((B, L, N), np.uint32),
+        "val": np.zeros((B, L, N), np.float32),
+        "counters": np.zeros((B, L, 3), np.uint64),
+    }
+    rc = lib().oracle_policy_scan(B, T, L, N, K, C, R, POLICIES[policy], lambda2, _ptr(p),
+                                  _ptr(res["topk"]), _ptr(res["misses"]), _ptr(res["proactive"]),
+                                  _ptr(res["cache_bits"]), _ptr(res["aux"]), _ptr(res["val"]),
+                                  _ptr(res["counters"]))
+    if rc != 0:
+        raise ValueError("oracle_policy_scan rejected the sizes")
+    return res
+
+
 class Chain:
     """State of one (stream, layer) chain for step-by-step replay."""
 

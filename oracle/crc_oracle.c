@@ -181,3 +181,194 @@ void oracle_metrics(double A, double D, double P, double T, double s_exp,
     *adj_hit = (A - D) / (A + P);
     *load_per_token = (D + P) * s_exp / T;
 }
+
+/* ------------------------------------------------------------------------ */
+/* comparison policies (Sec. 4 baselines "for cache update"; Sec. 4.3 and   */
+/* the appendix on ablations for Spatio-only)                               */
+/* ------------------------------------------------------------------------ */
+/*
+ * Readings (the paper names the classical policies and their references and
+ * gives LRFU's lambda = 0.5, nothing more):
+ *   - the classical policies (LRU, LFU, LRFU) only update the cache: no
+ *     pre-access refinement, no proactive load; each access demand-loads
+ *     S \ C in ascending expert index and, with the cache full, evicts the
+ *     member of V = C \ S with the lowest priority (ties: the highest index),
+ *     as Algorithm 1 does with s^T;
+ *   - LRU priority: the token index of the expert's last use;
+ *   - LFU priority: the number of accesses that selected the expert since it
+ *     entered the cache (1 on insertion);
+ *   - LRFU priority at token t: CRF * F(t - t_last), CRF updated at each use
+ *     to 1 + F(t - t_last) * CRF (1 on insertion), F(x) = 2^(-lambda x) with
+ *     lambda a multiple of 1/2, evaluated in fp32 as 2^(-q) (exact), times
+ *     fp32(2^(-1/2)) when lambda x is odd in halves, and 0 once q >= 126;
+ *   - Spatio-only: Algorithm 2's refinement with s^S = p^R_{t-1} + p^S_rho in
+ *     place of s^ST; an expert it loads counts as used at t; the demand loads
+ *     evict by LRU.
+ */
+enum { ORACLE_POLICY_LRU = 1, ORACLE_POLICY_LFU = 2, ORACLE_POLICY_LRFU = 3,
+       ORACLE_POLICY_SPATIO_LRU = 4 };
+
+static float lrfu_decay(int lambda2, long dt)        /* F(dt), lambda = lambda2 / 2 */
+{
+    const long halves = (long)lambda2 * dt;
+    const long q = halves / 2;
+    if (q >= 126) return 0.0f;
+    float f = ldexpf(1.0f, (int)-q);
+    if (halves % 2) f = f * 0.70710678118654752f;    /* fp32(2^(-1/2)) */
+    return f;
+}
+
+/* the member with the smallest integer priority, ties to the highest index */
+static int argmin_last_u32(const uint32_t *key, const uint8_t *member, int N)
+{
+    int v = -1;
+    for (int e = 0; e < N; e++)
+        if (member[e] && (v < 0 || key[e] <= key[v])) v = e;
+    return v;
+}
+
+/* One access of one chain under a comparison policy; fp32 throughout. */
+int oracle_policy_step(int N, int K, int C, int R, int policy, int lambda2, int t,
+                       const float *pR, const float *pS_pred, uint8_t *in_cache, int *count,
+                       uint32_t *aux, float *val, int *topk_out, int *misses_out,
+                       int *proactive_out)
+{
+    if (N < 1 || N > ORACLE_MAX_N || K < 1 || K > N || C < K || C > N || R < 0 ||
+        policy < ORACLE_POLICY_LRU || policy > ORACLE_POLICY_SPATIO_LRU || lambda2 < 0)
+        return -1;
+    int proactive = 0;
+    /* Spatio-only: pre-access refinement on s^S = p^R_{t-1} + p^S_rho */
+    if (policy == ORACLE_POLICY_SPATIO_LRU && R > 0 && t >= 1) {
+        float sS[ORACLE_MAX_N];
+        uint8_t before[ORACLE_MAX_N];
+        for (int e = 0; e < N; e++) {
+            sS[e] = val[e] + pS_pred[e];
+            before[e] = in_cache[e];
+        }
+        proactive = oracle_refine_f32(N, C, R, sS, in_cache, count, NULL);
+        for (int e = 0; e < N; e++)
+            if (in_cache[e] && !before[e]) aux[e] = (uint32_t)t;
+    }
+    /* native Top-K on p^R */
+    int ord[ORACLE_MAX_N];
+    order_desc_f32(pR, N, ord);
+    uint8_t inS[ORACLE_MAX_N], hit[ORACLE_MAX_N], inV[ORACLE_MAX_N];
+    memset(inS, 0, (size_t)N);
+    for (int k = 0; k < K; k++) {
+        topk_out[k] = ord[k];
+        inS[ord[k]] = 1;
+    }
+    for (int e = 0; e < N; e++) hit[e] = (uint8_t)(inS[e] && in_cache[e]);
+    /* the eviction priorities of this access (fixed while it inserts) */
+    uint32_t pri_u[ORACLE_MAX_N];
+    float pri_f[ORACLE_MAX_N];
+    for (int e = 0; e < N; e++) {
+        pri_u[e] = aux[e];
+        pri_f[e] = policy == ORACLE_POLICY_LRFU ? val[e] * lrfu_decay(lambda2, (long)t - (long)aux[e])
+                                                : 0.0f;
+    }
+    /* demand loads, ascending index; a full cache evicts argmin over C \ S */
+    int misses = 0;
+    for (int e = 0; e < N; e++) {
+        if (!inS[e] || in_cache[e]) continue;
+        misses++;
+        if (*count < C) {
+            in_cache[e] = 1;
+            (*count)++;
+            continue;
+        }
+        for (int u = 0; u < N; u++) inV[u] = (uint8_t)(in_cache[u] && !inS[u]);
+        int v = policy == ORACLE_POLICY_LRFU ? argmin_last_f32(pri_f, inV, N, NULL)
+                                             : argmin_last_u32(pri_u, inV, N);
+        in_cache[v] = 0;
+        in_cache[e] = 1;
+    }
+    /* the selected experts' priorities after the access */
+    for (int e = 0; e < N; e++) {
+        if (!inS[e]) continue;
+        if (policy == ORACLE_POLICY_LFU) {
+            aux[e] = hit[e] ? aux[e] + 1u : 1u;
+        } else if (policy == ORACLE_POLICY_LRFU) {
+            val[e] = hit[e] ? 1.0f + lrfu_decay(lambda2, (long)t - (long)aux[e]) * val[e] : 1.0f;
+            aux[e] = (uint32_t)t;
+        } else {
+            aux[e] = (uint32_t)t;
+        }
+    }
+    if (policy == ORACLE_POLICY_SPATIO_LRU)
+        for (int e = 0; e < N; e++) val[e] = pR[e];          /* p^R_{t-1} for the next access */
+    *misses_out = misses;
+    *proactive_out = proactive;
+    return 0;
+}
+
+/*
+ * Whole scan under a comparison policy: B streams, T tokens, L layers, cold
+ * start, fp32 probabilities [B][T][L][3][N] (p^S read by Spatio-only only).
+ * Outputs as oracle_scan (any trace pointer may be NULL), plus the per-expert
+ * policy state of the last token: aux_out [B][L][N] (LRU and Spatio-only:
+ * token of last use; LFU: count; LRFU: token of last use) and val_out
+ * [B][L][N] (LRFU: CRF; Spatio-only: p^R of the last token; else 0).
+ */
+int oracle_policy_scan(int B, int T, int L, int N, int K, int C, int R, int policy,
+                       int lambda2, const float *probs, uint8_t *topk, uint8_t *misses,
+                       uint8_t *proactive, uint32_t *cache_bits, uint32_t *aux_out,
+                       float *val_out, uint64_t *counters)
+{
+    if (B < 0 || T < 0 || L < 1 || N < 1 || N > ORACLE_MAX_N || K < 1 || K > N || C < K ||
+        C > N || R < 0)
+        return -1;
+    const size_t row = (size_t)3 * N;
+    uint8_t *in_cache = (uint8_t *)calloc((size_t)L * N, 1);
+    int *count = (int *)calloc((size_t)L, sizeof(int));
+    uint32_t *aux = (uint32_t *)calloc((size_t)L * N, sizeof(uint32_t));
+    float *val = (float *)calloc((size_t)L * N, sizeof(float));
+    int tk[ORACLE_MAX_N], rc = 0;
+    for (int b = 0; b < B && rc == 0; b++) {
+        memset(in_cache, 0, (size_t)L * N);
+        memset(count, 0, sizeof(int) * (size_t)L);
+        memset(aux, 0, sizeof(uint32_t) * (size_t)L * N);
+        memset(val, 0, sizeof(float) * (size_t)L * N);
+        uint64_t *ctr = counters + (size_t)b * L * 3;
+        memset(ctr, 0, sizeof(uint64_t) * (size_t)L * 3);
+        for (int t = 0; t < T && rc == 0; t++) {
+            for (int l = 0; l < L; l++) {
+                const size_t unit = ((size_t)b * T + t) * L + l;
+                const float *pR = probs + unit * row;
+                const float *pS = NULL;                     /* p^S_{rho(t,l)} */
+                if (l > 0)
+                    pS = probs + (unit - 1) * row + 2 * N;
+                else if (t > 0)
+                    pS = probs + (((size_t)b * T + (t - 1)) * L + (L - 1)) * row + 2 * N;
+                int mi, pr;
+                if (oracle_policy_step(N, K, C, R, policy, lambda2, t, pR, pS,
+                                       in_cache + (size_t)l * N, &count[l], aux + (size_t)l * N,
+                                       val + (size_t)l * N, tk, &mi, &pr) != 0) {
+                    rc = -1;
+                    break;
+                }
+                ctr[l * 3 + 0] += (uint64_t)(K - mi);
+                ctr[l * 3 + 1] += (uint64_t)mi;
+                ctr[l * 3 + 2] += (uint64_t)pr;
+                if (topk)
+                    for (int k = 0; k < K; k++) topk[unit * K + k] = (uint8_t)tk[k];
+                if (misses) misses[unit] = (uint8_t)mi;
+                if (proactive) proactive[unit] = (uint8_t)pr;
+            }
+        }
+        const int NW = (N + 31) / 32;
+        for (int l = 0; l < L; l++) {
+            uint32_t *bits = cache_bits + ((size_t)b * L + l) * NW;
+            memset(bits, 0, sizeof(uint32_t) * (size_t)NW);
+            for (int e = 0; e < N; e++)
+                if (in_cache[(size_t)l * N + e]) bits[e / 32] |= 1u << (e % 32);
+            if (aux_out) memcpy(aux_out + ((size_t)b * L + l) * N, aux + (size_t)l * N, 4 * (size_t)N);
+            if (val_out) memcpy(val_out + ((size_t)b * L + l) * N, val + (size_t)l * N, 4 * (size_t)N);
+        }
+    }
+    free(in_cache);
+    free(count);
+    free(aux);
+    free(val);
+    return rc;
+}
