@@ -144,6 +144,37 @@ int crc_cache_scan(const crc_problem *p, const float *scores_dev, int32_t T,
                    void *state_dev, size_t state_bytes, const crc_trace *trace,
                    void *stream);
 
+/* Comparison policies of the paper's evaluation (Sec. 4: the cache-update
+ * baselines LRU, LFU and LRFU with lambda = 0.5; Sec. 4.3 and the ablation
+ * appendix: Spatio-only, i.e. Algorithm 2's refinement on
+ * s^S = p^R_{t-1} + p^S_rho with LRU eviction for demand misses). */
+enum { CRC_POLICY_LRU = 1, CRC_POLICY_LFU = 2, CRC_POLICY_LRFU = 3, CRC_POLICY_SPATIO_LRU = 4 };
+
+/* The cache simulation of crc_cache_scan under a comparison policy, same
+ * arguments plus:
+ *   policy         one of CRC_POLICY_*; a state belongs to the policy of its
+ *                  first call (a later call with another policy, or a call of
+ *                  crc_cache_scan / crc_route_and_cache on it, latches
+ *                  CRC_ESTATE);
+ *   lambda_halves  LRFU's lambda in halves (0..8; 1 = the paper's 0.5),
+ *                  ignored by the other policies.
+ * LRU, LFU and LRFU demand-load S \ C and, with the cache full, evict the
+ * resident outside S with the lowest priority (token of last use; accesses
+ * since insertion; CRF * 2^(-lambda (t - t_last)) with the CRF updated to
+ * 1 + 2^(-lambda (t - t_last)) CRF at each use), ties to the highest expert
+ * index; they make no proactive load.  R is used by Spatio-only only.
+ * CRC_EINVAL for a policy or lambda outside these ranges. */
+int crc_cache_scan_policy(const crc_problem *p, const float *scores_dev, int32_t T,
+                          void *state_dev, size_t state_bytes, const crc_trace *trace,
+                          int32_t policy, int32_t lambda_halves, void *stream);
+
+/* Synchronises `stream` and copies a comparison policy's integer priorities
+ * [B][L][N] (LRU, Spatio-only, LRFU: token of last use; LFU: accesses since
+ * insertion) into aux_host; its float priorities (LRFU: CRF; Spatio-only:
+ * p^R of the last token) come with crc_state_read's retention array. */
+int crc_state_read_aux(const crc_problem *p, const void *state_dev, size_t state_bytes,
+                       uint32_t *aux_host, void *stream);
+
 /* Bytes of workspace crc_route_and_cache uses to process `chunk_tokens`
  * tokens per pass (the router scores of one chunk). */
 size_t crc_workspace_bytes(const crc_problem *p, int32_t chunk_tokens);

@@ -72,6 +72,9 @@ EXPORTS = [
     ("crc_route_and_cache_noalloc", ctypes.c_int,
      [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P]),
     ("crc_device_error", ctypes.c_int, []),
+    ("crc_cache_scan_policy", ctypes.c_int,
+     [PP, P, I32, P, SZ, ctypes.POINTER(crc_trace), I32, I32, P]),
+    ("crc_state_read_aux", ctypes.c_int, [PP, P, SZ, P, P]),
     ("crc_launch_count", U64, []),
     ("crc_strerror", ctypes.c_char_p, [ctypes.c_int]),
     ("crc_profile_begin", ctypes.c_int, []),
@@ -166,6 +169,27 @@ def crc_cache_scan(p: crc_problem, scores_ptr: int, T: int, state_ptr: int, stat
     _ck(load().crc_cache_scan(ctypes.byref(p), scores_ptr, T, state_ptr, state_bytes,
                               None if trace is None else ctypes.byref(trace), _stream(stream)),
         "crc_cache_scan")
+
+
+# comparison policies (crc.h CRC_POLICY_*)
+POLICIES = {"lru": 1, "lfu": 2, "lrfu": 3, "spatio_lru": 4}
+
+
+def crc_cache_scan_policy(p: crc_problem, scores_ptr: int, T: int, state_ptr: int,
+                          state_bytes: int, trace: crc_trace | None, policy: int,
+                          lambda_halves: int = 1, stream=None):
+    _ck(load().crc_cache_scan_policy(ctypes.byref(p), scores_ptr, T, state_ptr, state_bytes,
+                                     None if trace is None else ctypes.byref(trace), policy,
+                                     lambda_halves, _stream(stream)),
+        "crc_cache_scan_policy")
+
+
+def crc_state_read_aux(p: crc_problem, state_ptr: int, state_bytes: int,
+                       stream=None) -> np.ndarray:
+    aux = np.zeros((p.B, p.L, p.N), np.uint32)
+    _ck(load().crc_state_read_aux(ctypes.byref(p), state_ptr, state_bytes, aux.ctypes.data,
+                                  _stream(stream)), "crc_state_read_aux")
+    return aux
 
 
 def crc_workspace_bytes(p: crc_problem, chunk_tokens: int) -> int:
@@ -263,6 +287,9 @@ class State:
     def read(self, stream=None, **kw) -> dict:
         return crc_state_read(self.p, self.ptr, self.nbytes, stream, **kw)
 
+    def read_aux(self, stream=None) -> np.ndarray:
+        return crc_state_read_aux(self.p, self.ptr, self.nbytes, stream)
+
 
 @dataclass
 class Trace:
@@ -294,6 +321,15 @@ def cache_scan(p: crc_problem, scores, state: State, trace: Trace | None = None,
     T = scores.shape[1]
     crc_cache_scan(p, scores.data_ptr(), T, state.ptr, state.nbytes,
                    None if trace is None else trace.c(), stream)
+
+
+def cache_scan_policy(p: crc_problem, scores, state: State, policy, trace: Trace | None = None,
+                      lambda_halves: int = 1, stream=None):
+    """crc_cache_scan_policy: policy is a CRC_POLICY_* value or one of POLICIES."""
+    T = scores.shape[1]
+    code = POLICIES[policy] if isinstance(policy, str) else int(policy)
+    crc_cache_scan_policy(p, scores.data_ptr(), T, state.ptr, state.nbytes,
+                          None if trace is None else trace.c(), code, lambda_halves, stream)
 
 
 def route_and_cache(p: crc_problem, hidden, w_cat, state: State, trace: Trace | None = None,

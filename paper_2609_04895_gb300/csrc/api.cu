@@ -193,6 +193,37 @@ int crc_cache_scan(const crc_problem* p, const float* scores_dev, int32_t T, voi
                        static_cast<cudaStream_t>(stream));
 }
 
+int crc_cache_scan_policy(const crc_problem* p, const float* scores_dev, int32_t T,
+                          void* state_dev, size_t state_bytes, const crc_trace* trace,
+                          int32_t policy, int32_t lambda_halves, void* stream) {
+    int rc = check_problem(p, false);
+    if (rc) return rc;
+    if ((rc = check_state(p, state_dev, state_bytes))) return rc;
+    if (policy < CRC_POLICY_LRU || policy > CRC_POLICY_SPATIO_LRU) return CRC_EINVAL;
+    if (lambda_halves < 0 || lambda_halves > 8) return CRC_EINVAL;
+    if (T < 0) return CRC_EINVAL;
+    if (T == 0) return CRC_OK;
+    if (!scores_dev || !aligned(scores_dev, 16)) return CRC_EINVAL;
+    if ((rc = check_trace(trace))) return rc;
+    return launch_policy_scan(*p, scores_dev, T, state_dev, trace, T, 0, policy, lambda_halves,
+                              static_cast<cudaStream_t>(stream));
+}
+
+int crc_state_read_aux(const crc_problem* p, const void* state_dev, size_t state_bytes,
+                       uint32_t* aux_host, void* stream) {
+    int rc = check_problem(p, false);
+    if (rc) return rc;
+    if ((rc = check_state(p, state_dev, state_bytes))) return rc;
+    if (!aux_host) return CRC_EINVAL;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return CRC_ECUDA;
+    const StateLayout lay = state_layout(p->B, p->L, p->N);
+    const uint8_t* base = static_cast<const uint8_t*>(state_dev);
+    if (cudaMemcpy(aux_host, base + lay.aux, (size_t)p->B * p->L * p->N * sizeof(uint32_t),
+                   cudaMemcpyDeviceToHost) != cudaSuccess)
+        return CRC_ECUDA;
+    return CRC_OK;
+}
+
 size_t crc_fused_workspace_bytes(const crc_problem* p) {
     if (check_problem(p, true) != CRC_OK) return 0;
     return fused_workspace_bytes(*p);

@@ -296,19 +296,23 @@ __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, ui
 // the Spatio prediction of the predecessor and the native Top-K set `sel`
 // (this lane's V bits).  Updates the chain registers; returns the number of
 // proactive loads and writes the demand misses to *n_miss.
+// Algorithm 2's pre-access refinement of the chain's cache with priorities
+// a[e] + pS[e] (s^ST for the method, s^S for the Spatio-only ablation): the
+// top-R candidates in order, each skipped when resident, loaded into a free
+// slot, or swapped for the lowest resident when strictly higher.  Returns the
+// proactive loads.
 template <int V, bool ALL_VALID>
-__device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V],
-                                          const float (&pS)[V], bool refine, uint32_t valid,
-                                          int lane, int K, int C, int R, uint32_t sel,
-                                          int* n_miss) {
+__device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V], uint32_t valid,
+                                           int lane, int C, int R) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
     int pro = 0;
-    if (refine) {
+    {
         uint32_t kS[V];
         uint32_t u = 0u;                                       // best key outside the cache
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-            kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;   // s^ST = a^T + p^S_rho
+            // s^ST = a^T + p^S_rho (a = s^T of the previous token; Spatio-only: p^R)
+            kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;
             if (!((cr.cache >> v) & 1u)) u = kS[v] > u ? kS[v] : u;
         }
         // When at least R experts score strictly above every non-resident one,
@@ -348,6 +352,15 @@ __device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V]
             }
         }
     }
+    return pro;
+}
+
+template <int V, bool ALL_VALID>
+__device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V],
+                                          const float (&pS)[V], bool refine, uint32_t valid,
+                                          int lane, int K, int C, int R, uint32_t sel,
+                                          int* n_miss) {
+    int pro = refine ? scan_refine<V, ALL_VALID>(cr, pS, valid, lane, C, R) : 0;
 
     // demand misses and UpdateCache (Algorithm 1)
     const uint32_t dem = sel & ~cr.cache;
@@ -449,7 +462,8 @@ __global__ void __launch_bounds__(128) cache_scan_kernel(ScanArgs a) {
     const bool active = chain < a.B * a.L;
 
     const bool hdr_ok = hdr->magic == kStateMagic && hdr->L == a.L && hdr->N == a.N &&
-                        hdr->K == a.K && hdr->C == a.C && hdr->R == a.R && hdr->B == a.B;
+                        hdr->K == a.K && hdr->C == a.C && hdr->R == a.R && hdr->B == a.B &&
+                        hdr->policy == 0u;
     const int64_t t0 = hdr->t_next;
     const uint32_t parity = hdr->parity;
 

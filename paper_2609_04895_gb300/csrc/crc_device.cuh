@@ -28,7 +28,8 @@ struct StateHeader {           // 256 bytes at offset 0
     uint32_t done;             // completion counter of the running scan grid
     int32_t L, N, K, C, R, B;  // the problem this state was made for
     uint64_t expert_bytes;
-    uint32_t pad[50];
+    uint32_t policy;           // 0: the method; else the comparison policy that owns the state
+    uint32_t pad[49];
 };
 static_assert(sizeof(StateHeader) == 256, "header size");
 
@@ -39,15 +40,19 @@ struct ChainState {            // 64 bytes per (stream, layer)
 static_assert(sizeof(ChainState) == 64, "chain size");
 
 struct StateLayout {
-    size_t chains, retention, carry, total;
+    size_t chains, retention, carry, aux, total;
 };
 
+// chains [B][L]; retention [B][L][N] fp32 (a^T; a comparison policy's float
+// priority); carry [2][B][N] fp32 (p^S handed to the next call's layer 0);
+// aux [B][L][N] u32 (a comparison policy's integer priority).
 __host__ __device__ inline StateLayout state_layout(int B, int L, int N) {
     StateLayout s;
     s.chains = 256;
     s.retention = s.chains + (size_t)B * L * sizeof(ChainState);
     s.carry = s.retention + (size_t)B * L * N * sizeof(float);
-    s.total = s.carry + (size_t)2 * B * N * sizeof(float);
+    s.aux = s.carry + (size_t)2 * B * N * sizeof(float);
+    s.total = s.aux + (size_t)B * L * N * sizeof(uint32_t);
     s.total = (s.total + 255) & ~(size_t)255;
     return s;
 }

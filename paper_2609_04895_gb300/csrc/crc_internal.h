@@ -55,6 +55,10 @@ int launch_fused_n32(const crc_problem& p, const uint16_t* hidden, const uint16_
                      void* state, void* workspace, cudaStream_t stream);
 int launch_fused_n64(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                      void* state, void* workspace, cudaStream_t stream);
+// Cache scan under a comparison policy (policy_scan.cuh).
+int launch_policy_scan(const crc_problem& p, const float* scores, int T, void* state,
+                       const crc_trace* trace, int trace_T, int trace_t0, int policy,
+                       int lambda2, cudaStream_t stream);
 int launch_fused_n128(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                       void* state, void* workspace, cudaStream_t stream);
 

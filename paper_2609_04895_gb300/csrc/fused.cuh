@@ -388,7 +388,8 @@ __global__ void __launch_bounds__(512, 1)
     uint32_t* err = &hdr->error;
     uint32_t* abort_flag = a.ctl + 1;
     const bool hdr_ok = hdr->magic == kStateMagic && hdr->L == a.L && hdr->N == a.N &&
-                        hdr->K == a.K && hdr->C == a.C && hdr->R == a.R && hdr->B == a.B;
+                        hdr->K == a.K && hdr->C == a.C && hdr->R == a.R && hdr->B == a.B &&
+                        hdr->policy == 0u;
     const int64_t t0g = hdr->t_next;
     const uint32_t parity = hdr->parity;
 

@@ -46,7 +46,8 @@ def test_struct_layouts_match_header(crc):
 def test_sizes(crc):
     p = crc.problem_of(S.QWEN3_30B)
     B, L, N = p.B, p.L, p.N
-    expect = 256 + B * L * 64 + B * L * N * 4 + 2 * B * N * 4
+    # header, chains, retention, p^S carry, a comparison policy's integer priorities
+    expect = 256 + B * L * 64 + B * L * N * 4 + 2 * B * N * 4 + B * L * N * 4
     assert crc.crc_state_bytes(p) == (expect + 255) // 256 * 256
     assert crc.crc_workspace_bytes(p, 16) == B * 16 * L * 3 * N * 4
     assert crc.crc_workspace_bytes(p, 0) == 0
@@ -90,6 +91,24 @@ def test_router_limits_and_pointer_checks(crc):
                                    None) == crc.CRC_EINVAL
     assert lib.crc_synth_hidden(1, 1, 1, 3, 0, 0, 0.5, 0.5, None, 16, 16, None) == crc.CRC_EINVAL
     assert lib.crc_synth_hidden(1, 1, 1, 4, 0, 0, 1.5, 0.5, None, 16, 16, None) == crc.CRC_EINVAL
+
+
+def test_policy_scan_argument_checks(crc):
+    lib = crc.load()
+    p = crc.problem_of(S.QWEN3_30B)
+    n = crc.crc_state_bytes(p)
+    scan = lambda policy, lam, T=4, scores=16: lib.crc_cache_scan_policy(   # noqa: E731
+        ctypes.byref(p), scores, T, 256, n, None, policy, lam, None)
+    assert scan(0, 1) == crc.CRC_EINVAL                     # the method itself: crc_cache_scan
+    assert scan(5, 1) == crc.CRC_EINVAL
+    assert scan(crc.POLICIES["lrfu"], -1) == crc.CRC_EINVAL
+    assert scan(crc.POLICIES["lrfu"], 9) == crc.CRC_EINVAL
+    assert scan(crc.POLICIES["lru"], 1, T=-1) == crc.CRC_EINVAL
+    assert scan(crc.POLICIES["lru"], 1, T=0) == crc.CRC_OK
+    assert scan(crc.POLICIES["lfu"], 1, scores=8) == crc.CRC_EINVAL
+    assert lib.crc_cache_scan_policy(ctypes.byref(p), 16, 4, 256, n - 256, None, 1, 1,
+                                     None) == crc.CRC_ESTATE
+    assert lib.crc_state_read_aux(ctypes.byref(p), 256, n, None, None) == crc.CRC_EINVAL
 
 
 def test_strerror(crc):
