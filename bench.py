@@ -57,6 +57,10 @@ def parse_args():
     ap.add_argument("--only", choices=["fused", "pair", "router", "scan"], default="fused",
                     help="fused: crc_route_and_cache as one fused kernel (default); pair: "
                          "crc_route_scores then crc_cache_scan; router / scan: one part alone")
+    ap.add_argument("--policy", choices=["method", "lru", "lfu", "lrfu", "spatio_lru"],
+                    default="method",
+                    help="with --only scan: time a comparison policy's scan "
+                         "(crc_cache_scan_policy, LRFU lambda 0.5) instead of the method's")
     return ap.parse_args()
 
 
@@ -327,7 +331,11 @@ def main():
             return
         st.init()
         if args.only == "scan":
-            C.crc_cache_scan(p, scores.data_ptr(), w.T, st.ptr, st.nbytes, None, stream)
+            if args.policy != "method":
+                C.crc_cache_scan_policy(p, scores.data_ptr(), w.T, st.ptr, st.nbytes, None,
+                                        C.POLICIES[args.policy], 1, stream)
+            else:
+                C.crc_cache_scan(p, scores.data_ptr(), w.T, st.ptr, st.nbytes, None, stream)
             return
         if args.only == "pair":
             C.crc_route_scores(p, hd.data_ptr(), Wd.data_ptr(), w.T, heads, scores.data_ptr(),
@@ -367,7 +375,11 @@ def main():
     units_all = w.units * world
     value = units_all / (ms_per_step / 1000.0)
 
-    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step)
+    # a comparison policy's scan reads p^R only (Spatio-only: and p^S)
+    scan_heads = heads if args.policy == "method" else (2 if args.policy == "spatio_lru" else 1)
+    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step, scan_heads)
+    if args.policy != "method" and roof.get("kernel") == "cache_scan_kernel":
+        roof["kernel"] = f"cache_scan_policy_kernel ({args.policy})"
 
     # end to end through the C ABI from pinned host memory
     e2e = None
@@ -388,7 +400,7 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic",
             "config": dict(workload_config(w, None if args.only == "fused" and not args.chunk
-                                           else chunk), path=args.only,
+                                           else chunk), path=args.only, policy=args.policy,
                            workspace_bytes=int(ws_bytes)),
             "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
@@ -401,7 +413,7 @@ def main():
     return 0
 
 
-def rooflines(kt, w, heads, steps, ms, ms_per_step):
+def rooflines(kt, w, heads, steps, ms, ms_per_step, scan_heads=None):
     """Roofline of the dominant kernel (timed live over the timed region) and of
     the whole path (max of flops at bf16 peak and bytes at HBM bandwidth)."""
     pk, pk_src = peaks()
@@ -410,7 +422,7 @@ def rooflines(kt, w, heads, steps, ms, ms_per_step):
     t_s = kt[dom]["ms"] / 1000.0
     if dom == "scan":
         flops = 0.0
-        bytes_ = 4.0 * heads * w.N * w.units * steps          # probabilities read once
+        bytes_ = 4.0 * (scan_heads or heads) * w.N * w.units * steps   # probabilities read once
         kname = "cache_scan_kernel"
     elif dom == "router":
         flops = 2.0 * w.d * heads * w.N * w.units * steps
