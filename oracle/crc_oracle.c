@@ -20,6 +20,10 @@
  *                  rho(t,1) = (t-1, L), rho(t,l) = (t, l-1)
  *                  top-R candidates, insert / replace-lowest        (Algorithm 2)
  *   accounting     accesses, demand misses D, proactive loads P   (Sec. 4.1)
+ *   coverage loss  m_e = sigmoid((s_e - theta_B(s)) / tau),
+ *                  l(s, q) = sum_e q_e (1 - m_e), l^T and l^ST, their means
+ *                  and the gradient into the three heads' logits
+ *                                                            (Sec. 3.1-3.4)
  *
  * Readings where the paper is silent (each one is listed in the design notes):
  *   - one total order everywhere: score descending, expert index ascending.
@@ -371,4 +375,110 @@ int oracle_policy_scan(int B, int T, int L, int N, int K, int C, int R, int poli
     free(aux);
     free(val);
     return rc;
+}
+
+/* ------------------------------------------------------------------------ */
+/* soft Top-B cache-coverage losses (Sec. 3.1, 3.2, 3.3)                    */
+/* ------------------------------------------------------------------------ */
+/*
+ * For a priority s over N experts and a target distribution q:
+ *   theta_B(s) = the B-th largest entry of s,
+ *   m_e(s)     = sigmoid((s_e - theta_B(s)) / tau),
+ *   l(s, q)    = sum_e q_e (1 - m_e(s)).
+ * Temporal:        l^T_{t,l}  = l(s^T_{t,l}, p^R_{t+1,l}),  s^T = p^R + p^T,
+ *                  valid for t < T - 1 (a next-token target exists);
+ * Spatio-Temporal: l^ST_{t,l} = l(s^ST_{t,l}, p^R_{t,l}),
+ *                  s^ST = (p^R_{t-1,l} + p^T_{t-1,l}) + p^S_{rho(t,l)},
+ *                  valid for t >= 1 (a previous token and a predecessor exist).
+ * L_T, L_ST are the means over the valid positions of the B_s streams.
+ * Readings: the native distributions stay differentiable as targets too
+ * (Sec. 3.4), so d l / d q_e = 1 - m_e reaches the target's p^R; the
+ * subgradient of theta_B goes to the element at position B under the total
+ * order (score descending, index ascending); the priorities are formed in
+ * fp32 exactly as the GPU forms them (so both pick the same theta element),
+ * everything after that in fp64.
+ * Outputs: loss [B_s][T][L][2] (l^T, l^ST; 0 where invalid) and, if grad is
+ * not NULL, the gradient of w_T L_T + w_ST L_ST with respect to the logits of
+ * the three heads, [B_s][T][L][3][N] (through p = softmax(z)).
+ */
+static double coverage_loss(int N, int Btop, double tau, const float *s, const float *q,
+                            double *g, double *gq)
+{
+    int ord[ORACLE_MAX_N];
+    order_desc_f32(s, N, ord);
+    const int estar = ord[Btop - 1];
+    const double theta = (double)s[estar];
+    double loss = 0.0, sum_dm = 0.0;
+    for (int e = 0; e < N; e++) {
+        const double m = 1.0 / (1.0 + exp(-((double)s[e] - theta) / tau));
+        loss += (double)q[e] * (1.0 - m);
+        gq[e] = 1.0 - m;                                            /* d l / d q_e          */
+        const double dm = (double)q[e] * m * (1.0 - m) / tau;      /* q_e dm_e/dx_e / tau */
+        g[e] = -dm;                                                 /* d l / d s_e via s_e  */
+        sum_dm += dm;
+    }
+    g[estar] += sum_dm;                                             /* via theta = s_{e*}   */
+    return loss;
+}
+
+int oracle_cache_loss(int Bs, int T, int L, int N, int Btop, double tau, double w_T, double w_ST,
+                      const float *probs, float *loss_out, double *grad)
+{
+    if (Bs < 1 || T < 1 || L < 1 || N < 1 || N > ORACLE_MAX_N || Btop < 1 || Btop > N ||
+        !(tau > 0.0))
+        return -1;
+    const size_t row = (size_t)3 * N;
+    const size_t units = (size_t)Bs * T * L;
+    double *dp = (double *)calloc(units * row, sizeof(double));   /* d objective / d p */
+    double g[ORACLE_MAX_N], gq[ORACLE_MAX_N];
+    float sv[ORACLE_MAX_N];
+    const double nT = (double)Bs * (T - 1) * L, nST = (double)Bs * (T - 1) * L;
+    const double cT = nT > 0 ? w_T / nT : 0.0, cST = nST > 0 ? w_ST / nST : 0.0;
+    for (int b = 0; b < Bs; b++)
+        for (int t = 0; t < T; t++)
+            for (int l = 0; l < L; l++) {
+                const size_t u = ((size_t)b * T + t) * L + l;
+                const float *p = probs + u * row;
+                float *lo = loss_out + u * 2;
+                lo[0] = lo[1] = 0.0f;
+                if (t + 1 < T) {                                    /* l^T_{t,l} */
+                    const size_t uq = u + (size_t)L;                /* (t+1, l) */
+                    const float *q = probs + uq * row;              /* p^R_{t+1,l} */
+                    for (int e = 0; e < N; e++) sv[e] = p[e] + p[N + e];
+                    lo[0] = (float)coverage_loss(N, Btop, tau, sv, q, g, gq);
+                    for (int e = 0; e < N; e++) {
+                        dp[u * row + e] += cT * g[e];               /* p^R_{t,l} */
+                        dp[u * row + N + e] += cT * g[e];           /* p^T_{t,l} */
+                        dp[uq * row + e] += cT * gq[e];             /* target p^R_{t+1,l} */
+                    }
+                }
+                if (t >= 1) {                                       /* l^ST_{t,l} */
+                    const size_t up = u - (size_t)L;                /* (t-1, l) */
+                    const size_t ur = l > 0 ? u - 1 : (((size_t)b * T + (t - 1)) * L + (L - 1));
+                    const float *pp = probs + up * row, *pr = probs + ur * row;
+                    for (int e = 0; e < N; e++) {
+                        const float a = pp[e] + pp[N + e];
+                        sv[e] = a + pr[2 * N + e];
+                    }
+                    lo[1] = (float)coverage_loss(N, Btop, tau, sv, p, g, gq);   /* q = p^R_{t,l} */
+                    for (int e = 0; e < N; e++) {
+                        dp[up * row + e] += cST * g[e];             /* p^R_{t-1,l} */
+                        dp[up * row + N + e] += cST * g[e];         /* p^T_{t-1,l} */
+                        dp[ur * row + 2 * N + e] += cST * g[e];     /* p^S_{rho(t,l)} */
+                        dp[u * row + e] += cST * gq[e];             /* target p^R_{t,l} */
+                    }
+                }
+            }
+    if (grad) {                                 /* through each head's softmax: dz = p (dp - <p, dp>) */
+        for (size_t u = 0; u < units; u++)
+            for (int h = 0; h < 3; h++) {
+                const float *p = probs + u * row + (size_t)h * N;
+                const double *d = dp + u * row + (size_t)h * N;
+                double dot = 0.0;
+                for (int e = 0; e < N; e++) dot += (double)p[e] * d[e];
+                for (int e = 0; e < N; e++) grad[u * row + (size_t)h * N + e] = (double)p[e] * (d[e] - dot);
+            }
+    }
+    free(dp);
+    return 0;
 }
