@@ -54,9 +54,17 @@ def parse_args():
                     help="proactive-load bound R (default: the workload's; the large shape takes 2 or 8)")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override T (a smaller case, e.g. for an ncu capture)")
-    ap.add_argument("--only", choices=["fused", "pair", "router", "scan"], default="fused",
+    ap.add_argument("--only", choices=["fused", "pair", "router", "scan", "loss"], default="fused",
                     help="fused: crc_route_and_cache as one fused kernel (default); pair: "
-                         "crc_route_scores then crc_cache_scan; router / scan: one part alone")
+                         "crc_route_scores then crc_cache_scan; router / scan: one part alone; "
+                         "loss: the soft Top-B coverage losses and their gradient "
+                         "(crc_cache_loss) on the router's probabilities")
+    ap.add_argument("--top-b", type=int, default=0,
+                    help="with --only loss: B of the soft Top-B loss (0 = the paper's: 20 for "
+                         "N = 128, 8 for N = 32)")
+    ap.add_argument("--tau", type=float, default=0.0,
+                    help="with --only loss: temperature (0 = the paper's: 0.03 for N = 128, "
+                         "0.05 for N = 32)")
     ap.add_argument("--policy", choices=["method", "lru", "lfu", "lrfu", "spatio_lru"],
                     default="method",
                     help="with --only scan: time a comparison policy's scan "
@@ -241,11 +249,201 @@ def workload_of(args):
     return w
 
 
+LOSS_METRIC = "stream-token-layer coverage-loss units/sec (forward + gradient)"
+LOSS_UNIT = "units/s"
+
+
+def loss_settings(args, w):
+    """(B, tau) of the soft Top-B loss: the paper's main settings by backbone."""
+    top_b = args.top_b or (20 if w.N >= 128 else 8)
+    tau = args.tau or (0.03 if w.N >= 128 else 0.05)
+    return min(top_b, w.N), tau
+
+
+def loss_workload_config(w, top_b, tau):
+    cfg = workload_config(w)
+    cfg.update({"top_b": top_b, "tau": tau, "w_T": 1.0, "w_ST": 1.0,
+                "inputs": "router probabilities [B][T][L][3][N] fp32 from the router GEMM on "
+                          "the synthetic hidden states (untimed)",
+                "l2": "inputs larger than L2 (probabilities %.1f GB per step), no flush"
+                      % (12.0 * w.N * w.units / 1e9)})
+    return cfg
+
+
+def loss_oracle_sample(w, top_b, tau, seconds):
+    """Times oracle.cache_loss (as it stands, one thread) on the first tokens
+    of one stream: synthetic distributions of the workload's shape."""
+    import oracle
+    oracle.build()
+    nt = 8
+    while True:
+        pb = S.distributions(1, nt, w.L, w.N, seed=0)
+        t0 = time.perf_counter()
+        oracle.cache_loss(pb, top_b, tau)
+        dt = time.perf_counter() - t0
+        if dt * 4 > seconds or nt >= w.T:
+            break
+        nt = min(w.T, max(nt * 2, int(nt * seconds / max(dt, 1e-3) / 2)))
+    units = nt * w.L
+    return {"value": units / dt, "unit": LOSS_UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"1 stream x {nt} tokens x {w.L} layers = {units} units (fp64 losses and "
+                      f"logit gradient), {dt:.1f} s wall"}, units, dt
+
+
+def run_reference_loss(args, w):
+    import oracle
+    oracle.build()
+    top_b, tau = loss_settings(args, w)
+    budget = max(1.0, min(6.0, 150.0 / max(1, args.steps + args.warmup)))
+    _, units, dt = loss_oracle_sample(w, top_b, tau, budget)
+    nt = units // w.L
+    pb = S.distributions(1, nt, w.L, w.N, seed=0)
+    for _ in range(args.warmup):
+        oracle.cache_loss(pb, top_b, tau)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.cache_loss(pb, top_b, tau)
+    dt = time.perf_counter() - t0
+    value = units * args.steps / dt
+    line = {
+        "metric": LOSS_METRIC, "value": value, "unit": LOSS_UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": dict(loss_workload_config(w, top_b, tau),
+                       inputs="seeded synthetic distributions of the same shape (host)"),
+        "impl": "reference",
+        "cpu_baseline": {"value": value, "unit": LOSS_UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"1 stream x {nt} tokens x {w.L} layers = {units} units "
+                                   f"per step"},
+        "e2e": {"value": value, "unit": LOSS_UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_loss(args, P, C, w, p, dev, stream, rank, world):
+    """Times crc_cache_loss over the whole workload: per step, both coverage
+    losses at every (stream, token, layer), their means and the gradient with
+    respect to the three heads' logits.  The probabilities come from the
+    router GEMM on the synthetic hidden states (untimed)."""
+    import torch
+    import torch.distributed as dist
+    top_b, tau = loss_settings(args, w)
+    Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
+    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
+                           rho_l=w.rho_l, device=dev)
+    probs = P.route_scores(p, hd, Wd, heads=3)
+    del hd, Wd
+    loss = torch.empty((w.B, w.T, w.L, 2), dtype=torch.float32, device=dev)
+    means = torch.empty(2, dtype=torch.float64, device=dev)
+    grad = torch.empty_like(probs)
+    ws_bytes = C.crc_loss_workspace_bytes(p, w.T)
+    ws = torch.empty(max(ws_bytes, 256), dtype=torch.uint8, device=dev)
+
+    def step(src=probs):
+        C.crc_cache_loss(p, src.data_ptr(), w.T, 3, top_b, tau, 1.0, 1.0, loss.data_ptr(),
+                         means.data_ptr(), grad.data_ptr(), ws.data_ptr(), ws.numel(), stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    assert C.crc_device_error() == 0
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(gpu_id_for_smi(torch, dev.index or 0)) as clk:
+        C.crc_profile_begin()
+        n0 = C.crc_launch_count()
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        launches = C.crc_launch_count() - n0
+        kt = C.crc_profile_end()
+    ms = e0.elapsed_time(e1)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+    ms_per_step = ms / args.steps
+    value = w.units * world / (ms_per_step / 1000.0)
+    L_T, L_ST = (float(x) for x in means.cpu())
+
+    # roofline of the loss kernel: probabilities read once, gradient and losses written once
+    pk, pk_src = peaks()
+    per_unit = 24.0 * w.N + 8.0
+    avg_ms = kt["loss"]["ms"] / max(1, kt["loss"]["launches"])
+    achieved = per_unit * w.units / (avg_ms / 1000.0) / 1e9
+    V = 1 if w.N <= 32 else 2 if w.N <= 64 else 4 if w.N <= 128 else 8
+    kname = f"cache_loss_kernel<{V}>"
+    tr, _ = committed_traffic(kname, w.name)
+    roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / pk["hbm_gbs"], "traffic": None if tr is None else tr * w.units,
+            "kernel": kname, "peak_source": f"{pk_src} (copy)", "avg_launch_ms": avg_ms,
+            "launches": kt["loss"]["launches"],
+            "share_of_step": kt["loss"]["ms"] / ms if ms else None,
+            "bytes_per_unit": per_unit}
+    kernels = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / args.steps}
+               for k, v in kt.items() if v["launches"]}
+
+    e2e = None
+    if not args.no_e2e:
+        # the public call from pinned host probabilities; the means come back
+        host = torch.empty(probs.shape, dtype=torch.float32, pin_memory=True)
+        host.copy_(probs)
+        out = torch.empty(2, dtype=torch.float64, pin_memory=True)
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        f0.record(stream)
+        for _ in range(args.steps):
+            probs.copy_(host, non_blocking=True)
+            step()
+            out.copy_(means, non_blocking=True)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        ems = f0.elapsed_time(f1)
+        if world > 1:
+            t = torch.tensor([ems], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        e2e = {"value": w.units * world / (ems / args.steps / 1000.0), "unit": LOSS_UNIT,
+               "h2d_bytes_per_step": int(probs.numel() * 4), "d2h_bytes_per_step": 16,
+               "ms_per_step": ems / args.steps}
+        del host
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        cpu, _, _ = loss_oracle_sample(w, top_b, tau, args.cpu_seconds)
+    if rank == 0:
+        line = {
+            "metric": LOSS_METRIC, "value": value, "unit": LOSS_UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": dict(loss_workload_config(w, top_b, tau), path="loss"),
+            "roofline": roof, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": int(launches), "clocks": clk.summary(),
+            "losses": {"L_T": L_T, "L_ST": L_ST},
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     w = workload_of(args)
+    if args.only == "loss":
+        return run_reference_loss(args, w)
     import oracle
     oracle.build()
     threads = oracle.default_threads()
@@ -306,6 +504,8 @@ def main():
     heads = 3 if w.R > 0 else 2
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream()
+    if args.only == "loss":
+        return run_loss(args, P, C, w, p, dev, stream, rank, world)
     if 2 * w.B * w.T * w.L * w.d > STREAM_BYTES:
         return run_streamed(args, P, C, w, p, heads, dev, stream, rank, world)
 

@@ -264,3 +264,32 @@ def near_uniform_scores(shape, seed: int, lo: float = 1e-6) -> np.ndarray:
     u[0::2] = (w0 >> 8).astype(np.float64) / 16777216.0
     u[1::2] = (w2 >> 8).astype(np.float64) / 16777216.0
     return np.maximum(u[:n], lo).astype(np.float32).reshape(shape)
+
+
+def distributions(B: int, T: int, L: int, N: int, seed: int, rho: float = 0.6,
+                  power: float = 20.0, quant: int | None = None, streams=None) -> np.ndarray:
+    """Router-like probability rows fp32 [B][T][L][3][N] for exercising the
+    coverage losses alone (host PCG64, one generator per stream).
+
+    Each row is a normalised positive draw: x_t = rho x_{t-1} + (1 - rho) u_t^power
+    with u ~ U(0, 1) per (stream, token, layer, head, expert), so a few experts
+    dominate each row and neighbouring tokens stay similar, then p = x / sum x.
+    quant rounds to multiples of 1/quant afterwards (ties on purpose).  streams
+    selects a subset of the B streams (the same rows as in the full draw).
+    With the defaults at N = 128 the top 8 experts hold about 0.36 of a row's
+    mass and consecutive tokens correlate at about 0.6."""
+    idx = range(B) if streams is None else streams
+    out = np.empty((len(idx), T, L, 3, N), np.float32)
+    for i, b in enumerate(idx):
+        rng = np.random.default_rng([seed, b])
+        u = rng.random((T, L, 3, N), dtype=np.float32) ** np.float32(power)
+        x = np.empty_like(u)
+        x[0] = u[0]
+        for t in range(1, T):
+            x[t] = np.float32(rho) * x[t - 1] + np.float32(1.0 - rho) * u[t]
+        x += np.float32(1e-6)
+        x /= x.sum(-1, keepdims=True)
+        if quant:
+            x = np.round(x * quant) / np.float32(quant)
+        out[i] = x
+    return out

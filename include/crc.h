@@ -237,6 +237,41 @@ int crc_route_and_cache_noalloc(const crc_problem *p, const uint16_t *hidden_dev
 /* Support                                                                  */
 /* ------------------------------------------------------------------------ */
 
+/* Soft Top-B cache-coverage losses and their gradient (Sec. 3.1-3.4): the
+ * training objective of the Temporal and Spatio heads, over whole sequences
+ * (tokens 0 .. T-1 of every stream).  With theta_B(s) the top_b-th largest
+ * entry of s, m_e(s) = sigmoid((s_e - theta_B(s)) / tau) and
+ * l(s, q) = sum_e q_e (1 - m_e(s)):
+ *   l^T_{t,l}  = l(p^R_{t,l} + p^T_{t,l}, p^R_{t+1,l})                  t < T-1
+ *   l^ST_{t,l} = l(p^R_{t-1,l} + p^T_{t-1,l} + p^S_{rho(t,l)}, p^R_{t,l}) t >= 1
+ *   L_T, L_ST  = their means over the B (T-1) L valid positions each.
+ * The priorities are summed in fp32 in that order (as the cache scan sums
+ * them), theta_B is exact on those fp32 values and its subgradient goes to
+ * the element at position top_b of the total order; the rest is fp32, the
+ * means are fp64 sums in a fixed order (no atomics: results are
+ * deterministic).
+ *   probs_dev   fp32 [B][T][L][3][N] (crc_route_scores' layout; finite,
+ *               >= 0), 16-byte aligned.  heads = 2 reads the R and T heads
+ *               only and computes l^T alone (l^ST = L_ST = 0, the S rows of
+ *               grad_dev untouched).
+ *   top_b       1..N;  tau > 0;  w_T, w_ST finite (the objective is
+ *               w_T L_T + w_ST L_ST).
+ *   loss_dev    fp32 [B][T][L][2]: l^T, l^ST per position (0 where not
+ *               valid), or NULL.
+ *   means_dev   fp64 [2] = (L_T, L_ST), or NULL.  Needs workspace_dev with
+ *               crc_loss_workspace_bytes(p, T) bytes, 256-byte aligned.
+ *   grad_dev    fp32 [B][T][L][3][N], or NULL: the gradient of the objective
+ *               with respect to each head's logits z (p = softmax(z)); the
+ *               native distributions are differentiable both as priorities
+ *               and as targets.  16-byte aligned, not aliasing probs_dev.
+ * K, C and R of the problem are not used.  T = 0 is a no-op.  Device-side
+ * failures: crc_device_error(). */
+size_t crc_loss_workspace_bytes(const crc_problem *p, int32_t T);
+int crc_cache_loss(const crc_problem *p, const float *probs_dev, int32_t T, int32_t heads,
+                   int32_t top_b, double tau, double w_T, double w_ST, float *loss_dev,
+                   double *means_dev, float *grad_dev, void *workspace_dev,
+                   size_t workspace_bytes, void *stream);
+
 /* Synchronises the device and returns (then clears) the error latched by
  * calls without a state (crc_route_scores), CRC_OK if none. */
 int crc_device_error(void);
@@ -252,7 +287,8 @@ uint64_t crc_launch_count(void);
  * bookkeeping only; off by default.  Not thread-safe against concurrent
  * library calls from other host threads. */
 enum { CRC_KERNEL_ROUTER = 0, CRC_KERNEL_SCAN = 1, CRC_KERNEL_STATE = 2, CRC_KERNEL_SYNTH = 3,
-       CRC_KERNEL_FUSED = 4, CRC_KERNEL_KINDS = 8 };
+       CRC_KERNEL_FUSED = 4, CRC_KERNEL_LOSS = 5, CRC_KERNEL_LOSS_MEANS = 6,
+       CRC_KERNEL_KINDS = 8 };
 typedef struct crc_kernel_times {
     uint64_t launches[CRC_KERNEL_KINDS];
     double ms[CRC_KERNEL_KINDS];

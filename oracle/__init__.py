@@ -180,23 +180,25 @@ def policy_scan(probs: np.ndarray, K: int, C: int, R: int, policy: str, lambda2:
 
 
 def cache_loss(probs: np.ndarray, top_b: int, tau: float, w_T: float = 1.0, w_ST: float = 1.0,
-               grad: bool = True) -> dict:
+               grad: bool = True, grad_p: bool = False) -> dict:
     """Soft Top-B coverage losses (Sec. 3.1-3.3) over fp32 probabilities
     [B][T][L][3][N]: per-unit l^T and l^ST [B][T][L][2], their means over the
     valid positions, and the gradient of w_T L_T + w_ST L_ST with respect to
     the three heads' logits [B][T][L][3][N] (fp64); the native distributions
-    are differentiable both as priorities and as targets (Sec. 3.4)."""
+    are differentiable both as priorities and as targets (Sec. 3.4).
+    grad_p adds the gradient with respect to the probabilities ("grad_p")."""
     p = np.ascontiguousarray(probs, dtype=np.float32)
     B, T, L, three, N = p.shape
     assert three == 3
     loss = np.zeros((B, T, L, 2), np.float32)
     g = np.zeros(p.shape, np.float64) if grad else None
+    gp = np.zeros(p.shape, np.float64) if grad_p else None
     rc = lib().oracle_cache_loss(B, T, L, N, top_b, ctypes.c_double(tau), ctypes.c_double(w_T),
-                                 ctypes.c_double(w_ST), _ptr(p), _ptr(loss), _ptr(g))
+                                 ctypes.c_double(w_ST), _ptr(p), _ptr(loss), _ptr(g), _ptr(gp))
     if rc != 0:
         raise ValueError("oracle_cache_loss rejected the sizes")
     n = B * (T - 1) * L
-    return {"loss": loss, "grad": g,
+    return {"loss": loss, "grad": g, "grad_p": gp,
             "L_T": float(loss[..., 0].astype(np.float64).sum() / n) if n else 0.0,
             "L_ST": float(loss[..., 1].astype(np.float64).sum() / n) if n else 0.0}
 

@@ -399,7 +399,8 @@ int oracle_policy_scan(int B, int T, int L, int N, int K, int C, int R, int poli
  * everything after that in fp64.
  * Outputs: loss [B_s][T][L][2] (l^T, l^ST; 0 where invalid) and, if grad is
  * not NULL, the gradient of w_T L_T + w_ST L_ST with respect to the logits of
- * the three heads, [B_s][T][L][3][N] (through p = softmax(z)).
+ * the three heads, [B_s][T][L][3][N] (through p = softmax(z)); if grad_p is not
+ * NULL, the gradient with respect to the probabilities, same layout.
  */
 static double coverage_loss(int N, int Btop, double tau, const float *s, const float *q,
                             double *g, double *gq)
@@ -422,7 +423,7 @@ static double coverage_loss(int N, int Btop, double tau, const float *s, const f
 }
 
 int oracle_cache_loss(int Bs, int T, int L, int N, int Btop, double tau, double w_T, double w_ST,
-                      const float *probs, float *loss_out, double *grad)
+                      const float *probs, float *loss_out, double *grad, double *grad_p)
 {
     if (Bs < 1 || T < 1 || L < 1 || N < 1 || N > ORACLE_MAX_N || Btop < 1 || Btop > N ||
         !(tau > 0.0))
@@ -469,6 +470,7 @@ int oracle_cache_loss(int Bs, int T, int L, int N, int Btop, double tau, double 
                     }
                 }
             }
+    if (grad_p) memcpy(grad_p, dp, units * row * sizeof(double));
     if (grad) {                                 /* through each head's softmax: dz = p (dp - <p, dp>) */
         for (size_t u = 0; u < units; u++)
             for (int h = 0; h < 3; h++) {

@@ -39,7 +39,8 @@ class crc_stats(ctypes.Structure):
                 ("error", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
 
 
-KERNEL_KINDS = {"router": 0, "scan": 1, "state": 2, "synth": 3, "fused": 4}
+KERNEL_KINDS = {"router": 0, "scan": 1, "state": 2, "synth": 3, "fused": 4, "loss": 5,
+                "loss_means": 6}
 
 
 class crc_kernel_times(ctypes.Structure):
@@ -75,6 +76,8 @@ EXPORTS = [
     ("crc_cache_scan_policy", ctypes.c_int,
      [PP, P, I32, P, SZ, ctypes.POINTER(crc_trace), I32, I32, P]),
     ("crc_state_read_aux", ctypes.c_int, [PP, P, SZ, P, P]),
+    ("crc_loss_workspace_bytes", SZ, [PP, I32]),
+    ("crc_cache_loss", ctypes.c_int, [PP, P, I32, I32, I32, D, D, D, P, P, P, P, SZ, P]),
     ("crc_launch_count", U64, []),
     ("crc_strerror", ctypes.c_char_p, [ctypes.c_int]),
     ("crc_profile_begin", ctypes.c_int, []),
@@ -190,6 +193,18 @@ def crc_state_read_aux(p: crc_problem, state_ptr: int, state_bytes: int,
     _ck(load().crc_state_read_aux(ctypes.byref(p), state_ptr, state_bytes, aux.ctypes.data,
                                   _stream(stream)), "crc_state_read_aux")
     return aux
+
+
+def crc_loss_workspace_bytes(p: crc_problem, T: int) -> int:
+    return int(load().crc_loss_workspace_bytes(ctypes.byref(p), T))
+
+
+def crc_cache_loss(p: crc_problem, probs_ptr: int, T: int, heads: int, top_b: int, tau: float,
+                   w_T: float, w_ST: float, loss_ptr, means_ptr, grad_ptr, ws_ptr, ws_bytes: int,
+                   stream=None):
+    _ck(load().crc_cache_loss(ctypes.byref(p), probs_ptr, T, heads, top_b, tau, w_T, w_ST,
+                              loss_ptr, means_ptr, grad_ptr, ws_ptr, ws_bytes, _stream(stream)),
+        "crc_cache_loss")
 
 
 def crc_workspace_bytes(p: crc_problem, chunk_tokens: int) -> int:
@@ -330,6 +345,31 @@ def cache_scan_policy(p: crc_problem, scores, state: State, policy, trace: Trace
     code = POLICIES[policy] if isinstance(policy, str) else int(policy)
     crc_cache_scan_policy(p, scores.data_ptr(), T, state.ptr, state.nbytes,
                           None if trace is None else trace.c(), code, lambda_halves, stream)
+
+
+def cache_loss(p: crc_problem, probs, top_b: int, tau: float, w_T: float = 1.0,
+               w_ST: float = 1.0, heads: int = 3, grad: bool = True, loss=None, means=None,
+               grad_out=None, workspace=None, stream=None):
+    """crc_cache_loss over probs [B][T][L][3][N] (fp32, on the device).
+
+    Returns (loss [B][T][L][2] fp32, means [2] fp64 = (L_T, L_ST), grad
+    [B][T][L][3][N] fp32 or None); pass preallocated tensors to reuse them."""
+    import torch
+    B, T, L, H, N = probs.shape
+    dev = probs.device
+    if loss is None:
+        loss = torch.empty((B, T, L, 2), dtype=torch.float32, device=dev)
+    if means is None:
+        means = torch.empty(2, dtype=torch.float64, device=dev)
+    if grad and grad_out is None:
+        grad_out = torch.zeros((B, T, L, 3, N), dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = torch.empty(max(crc_loss_workspace_bytes(p, T), 256), dtype=torch.uint8,
+                                device=dev)
+    crc_cache_loss(p, probs.data_ptr(), T, heads, top_b, tau, w_T, w_ST, loss.data_ptr(),
+                   means.data_ptr(), grad_out.data_ptr() if grad else None, workspace.data_ptr(),
+                   workspace.numel(), stream)
+    return loss, means, (grad_out if grad else None)
 
 
 def route_and_cache(p: crc_problem, hidden, w_cat, state: State, trace: Trace | None = None,

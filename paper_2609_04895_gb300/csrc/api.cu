@@ -1,6 +1,7 @@
 // C-ABI entry points of the library (declared in include/crc.h): argument
 // validation, state handling and the route-and-cache driver.
 #include <atomic>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -266,6 +267,38 @@ int crc_route_and_cache(const crc_problem* p, const uint16_t* hidden_dev,
         if ((rc = launch_scan(*p, scores, n, state_dev, trace, T, t0, s))) return rc;
     }
     return CRC_OK;
+}
+
+size_t crc_loss_workspace_bytes(const crc_problem* p, int32_t T) {
+    if (check_problem(p, false) != CRC_OK || T < 1) return 0;
+    const LossPlan pl = loss_plan(p->B, p->L, T);
+    const size_t bytes = (size_t)p->B * p->L * pl.nchunks * 2 * sizeof(double);
+    return (bytes + 255) / 256 * 256;
+}
+
+int crc_cache_loss(const crc_problem* p, const float* probs_dev, int32_t T, int32_t heads,
+                   int32_t top_b, double tau, double w_T, double w_ST, float* loss_dev,
+                   double* means_dev, float* grad_dev, void* workspace_dev,
+                   size_t workspace_bytes, void* stream) {
+    int rc = check_problem(p, false);
+    if (rc) return rc;
+    if (T < 0 || (heads != 2 && heads != 3)) return CRC_EINVAL;
+    if (top_b < 1 || top_b > p->N) return CRC_EINVAL;
+    if (!(tau > 0.0) || !std::isfinite(tau) || !std::isfinite(1.0 / tau)) return CRC_EINVAL;
+    if (!std::isfinite(w_T) || !std::isfinite(w_ST)) return CRC_EINVAL;
+    if (T == 0) return CRC_OK;
+    if (!probs_dev || !aligned(probs_dev, 16)) return CRC_EINVAL;
+    if (grad_dev && (!aligned(grad_dev, 16) || (const void*)grad_dev == (const void*)probs_dev))
+        return CRC_EINVAL;
+    if (loss_dev && !aligned(loss_dev, 4)) return CRC_EINVAL;
+    if (means_dev) {
+        if (!aligned(means_dev, 8) || !workspace_dev || !aligned(workspace_dev, 256) ||
+            workspace_bytes < crc_loss_workspace_bytes(p, T))
+            return CRC_EINVAL;
+    }
+    if (!loss_dev && !means_dev && !grad_dev) return CRC_OK;
+    return launch_cache_loss(*p, probs_dev, T, heads, top_b, tau, w_T, w_ST, loss_dev, means_dev,
+                             grad_dev, workspace_dev, static_cast<cudaStream_t>(stream));
 }
 
 int crc_device_error(void) {

@@ -62,6 +62,16 @@ int launch_policy_scan(const crc_problem& p, const float* scores, int T, void* s
 int launch_fused_n128(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                       void* state, void* workspace, cudaStream_t stream);
 
+// Soft Top-B coverage losses (loss.cu): the task split over token chunks and
+// the launch; workspace = per-task sums, 16 bytes per task.
+struct LossPlan {
+    int nchunks, chunk;
+};
+LossPlan loss_plan(int B, int L, int T);
+int launch_cache_loss(const crc_problem& p, const float* probs, int T, int heads, int top_b,
+                      double tau, double w_T, double w_ST, float* loss, double* means,
+                      float* grad, void* workspace, cudaStream_t stream);
+
 int launch_state_init(const crc_problem& p, void* state, size_t bytes, cudaStream_t stream);
 
 int launch_synth_hidden(int B, int T, int L, int d, int t0, uint32_t seed, double rho_t,

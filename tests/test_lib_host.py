@@ -111,6 +111,33 @@ def test_policy_scan_argument_checks(crc):
     assert lib.crc_state_read_aux(ctypes.byref(p), 256, n, None, None) == crc.CRC_EINVAL
 
 
+def test_cache_loss_argument_checks(crc):
+    lib = crc.load()
+    p = crc.problem_of(S.QWEN3_30B)
+    # per-task fp64 sums: B * L tasks per token chunk, 3 chunks of 342 tokens at T = 1024
+    assert crc.crc_loss_workspace_bytes(p, 1024) == (64 * 48 * 3 * 16 + 255) // 256 * 256
+    assert crc.crc_loss_workspace_bytes(p, 0) == 0
+    ws = crc.crc_loss_workspace_bytes(p, 8)
+    call = lambda T=8, heads=3, top_b=20, tau=0.03, wT=1.0, wST=1.0, probs=256, loss=256, \
+        means=None, grad=None, ws_ptr=256, ws_bytes=ws: lib.crc_cache_loss(  # noqa: E731
+            ctypes.byref(p), probs, T, heads, top_b, tau, wT, wST, loss, means, grad, ws_ptr,
+            ws_bytes, None)
+    assert call(T=0) == crc.CRC_OK
+    assert call(T=-1) == crc.CRC_EINVAL
+    assert call(heads=1) == crc.CRC_EINVAL
+    assert call(top_b=0) == crc.CRC_EINVAL and call(top_b=129) == crc.CRC_EINVAL
+    assert call(tau=0.0) == crc.CRC_EINVAL and call(tau=float("nan")) == crc.CRC_EINVAL
+    assert call(tau=1e-320) == crc.CRC_EINVAL                 # 1 / tau overflows
+    assert call(wT=float("inf")) == crc.CRC_EINVAL
+    assert call(probs=None) == crc.CRC_EINVAL and call(probs=8) == crc.CRC_EINVAL
+    assert call(grad=256) == crc.CRC_EINVAL                   # aliases probs
+    assert call(grad=4104) == crc.CRC_EINVAL                  # misaligned
+    assert call(means=512, ws_bytes=ws - 1) == crc.CRC_EINVAL
+    assert call(means=512, ws_ptr=None) == crc.CRC_EINVAL
+    assert call(means=512, ws_ptr=128) == crc.CRC_EINVAL
+    assert call(loss=None) == crc.CRC_OK                      # nothing requested
+
+
 def test_strerror(crc):
     assert "unsupported" in crc.crc_strerror(2) or "limits" in crc.crc_strerror(2)
     assert crc.crc_strerror(99) == "unknown error code"
