@@ -173,10 +173,30 @@ def gpu_id_for_smi(torch, dev: int) -> str:
         return str(dev)
 
 
-def source_hash() -> str:
+# The sources each profiled kernel is built from: a committed traffic figure
+# stands only while none of them has changed.
+KERNEL_SOURCES = {
+    "fused": ["fused.cu", "fused.cuh", "fused_launch.cuh", "fused_n16.cu", "fused_n32.cu",
+              "fused_n64.cu", "fused_n128.cu", "router_gemm.cuh", "cache_scan.cuh",
+              "crc_device.cuh"],
+    "router": ["router.cu", "router_gemm.cuh", "crc_device.cuh"],
+    "scan": ["scan.cu", "cache_scan.cuh", "crc_device.cuh"],
+    "policy": ["policy.cu", "policy_scan.cuh", "cache_scan.cuh", "crc_device.cuh"],
+    "loss": ["loss.cu"],
+}
+
+
+def kernel_family(kernel: str) -> str:
+    for fam in ("policy", "fused", "router", "loss"):
+        if fam in kernel:
+            return fam
+    return "scan"
+
+
+def source_hash(kernel: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_04895_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in sorted(KERNEL_SOURCES[kernel_family(kernel)]):
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
@@ -191,7 +211,7 @@ def committed_traffic(kernel: str, workload: str):
     except (OSError, ValueError):
         return None, None
     e = d.get(kernel, {}).get(workload)
-    if not e or e.get("src_sha") != source_hash():
+    if not e or e.get("src_sha") != source_hash(kernel):
         return None, None
     return e.get("dram_bytes_per_unit"), e.get("source")
 
@@ -271,23 +291,24 @@ def loss_workload_config(w, top_b, tau):
 
 
 def loss_oracle_sample(w, top_b, tau, seconds):
-    """Times oracle.cache_loss (as it stands, one thread) on the first tokens
-    of one stream: synthetic distributions of the workload's shape."""
+    """Times oracle.cache_loss (as it stands, one thread) on the first streams
+    of the workload (whole sequences): synthetic distributions of its shape."""
     import oracle
     oracle.build()
-    nt = 8
-    while True:
-        pb = S.distributions(1, nt, w.L, w.N, seed=0)
-        t0 = time.perf_counter()
-        oracle.cache_loss(pb, top_b, tau)
-        dt = time.perf_counter() - t0
-        if dt * 4 > seconds or nt >= w.T:
-            break
-        nt = min(w.T, max(nt * 2, int(nt * seconds / max(dt, 1e-3) / 2)))
-    units = nt * w.L
+    pilot = S.distributions(1, min(64, w.T), w.L, w.N, seed=0)
+    t0 = time.perf_counter()
+    oracle.cache_loss(pilot, top_b, tau)
+    rate = pilot.shape[1] * w.L / max(time.perf_counter() - t0, 1e-6)     # units/s
+    nb = int(max(1, min(w.B, rate * seconds // (w.T * w.L))))
+    nt = w.T if nb > 1 or rate * seconds >= w.T * w.L else int(max(8, rate * seconds // w.L))
+    pb = S.distributions(nb, nt, w.L, w.N, seed=0)
+    t0 = time.perf_counter()
+    oracle.cache_loss(pb, top_b, tau)
+    dt = time.perf_counter() - t0
+    units = nb * nt * w.L
     return {"value": units / dt, "unit": LOSS_UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"1 stream x {nt} tokens x {w.L} layers = {units} units (fp64 losses and "
-                      f"logit gradient), {dt:.1f} s wall"}, units, dt
+            "sample": f"{nb} stream(s) x {nt} tokens x {w.L} layers = {units} units (fp64 "
+                      f"losses and logit gradient), {dt:.1f} s wall"}, units, dt
 
 
 def run_reference_loss(args, w):
@@ -296,8 +317,9 @@ def run_reference_loss(args, w):
     top_b, tau = loss_settings(args, w)
     budget = max(1.0, min(6.0, 150.0 / max(1, args.steps + args.warmup)))
     _, units, dt = loss_oracle_sample(w, top_b, tau, budget)
-    nt = units // w.L
-    pb = S.distributions(1, nt, w.L, w.N, seed=0)
+    nb = max(1, units // (w.T * w.L))
+    nt = units // (nb * w.L)
+    pb = S.distributions(nb, nt, w.L, w.N, seed=0)
     for _ in range(args.warmup):
         oracle.cache_loss(pb, top_b, tau)
     t0 = time.perf_counter()
@@ -314,8 +336,8 @@ def run_reference_loss(args, w):
                        inputs="seeded synthetic distributions of the same shape (host)"),
         "impl": "reference",
         "cpu_baseline": {"value": value, "unit": LOSS_UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"1 stream x {nt} tokens x {w.L} layers = {units} units "
-                                   f"per step"},
+                         "sample": f"{nb} stream(s) x {nt} tokens x {w.L} layers = {units} "
+                                   f"units per step"},
         "e2e": {"value": value, "unit": LOSS_UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }

@@ -48,14 +48,10 @@ struct LossArgs {
     float* grad;          // [B][T][L][3][N] or null
     double* partial;      // [tasks][2] per-task sums of l^T and l^ST, or null
     int B, T, L, N, heads, top_b, chunk, nchunks;
-    float inv_tau, cT, cST;
+    float k2;             // log2(e) / tau
+    float cT, cST;        // w_T / |Omega_T|, w_ST / |Omega_ST|: coefficients of dl/dq
+    float gT, gST;        // the same over tau: coefficients of -w (dl/ds = -w / tau)
 };
-
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
-    return v;
-}
 
 // Row element e = V * lane + j lives in slot j of `lane` (lanes >= N / V idle).
 template <int V>
@@ -140,6 +136,66 @@ __device__ __forceinline__ uint32_t theta_key(const uint32_t (&k)[V], bool valid
     return prefix;
 }
 
+// theta_B from a guess g (the same term's theta at the previous token, which
+// is close: consecutive tokens route alike).  With n = #{k >= g}, theta is
+// the (n - B + 1)-th smallest key >= g, or the (B - n)-th largest key < g;
+// those are taken one distinct value at a time (redux min / max, then the
+// count of that value, so ties count with their multiplicity).  More than
+// kExtract rounds, or a round without a candidate, falls back to the bit
+// search.  Exact either way.
+constexpr int kExtract = 6;
+
+template <int V>
+__device__ __forceinline__ uint32_t theta_near(const uint32_t (&k)[V], bool valid, int top_b,
+                                               uint32_t g) {
+    uint32_t c = 0;
+#pragma unroll
+    for (int j = 0; j < V; ++j) c += valid && k[j] >= g ? 1u : 0u;
+    const int n = (int)__reduce_add_sync(kFull, c);
+    if (n >= top_b) {
+        int r = n - top_b;                          // keys >= g that rank below theta
+        uint32_t lower = g;
+        if (r < kExtract) {
+#pragma unroll 1
+            for (int it = 0; it < kExtract; ++it) {
+                uint32_t m = 0xffffffffu;
+#pragma unroll
+                for (int j = 0; j < V; ++j) m = valid && k[j] >= lower && k[j] < m ? k[j] : m;
+                m = __reduce_min_sync(kFull, m);
+                uint32_t e = 0;
+#pragma unroll
+                for (int j = 0; j < V; ++j) e += valid && k[j] == m ? 1u : 0u;
+                const int ce = (int)__reduce_add_sync(kFull, e);
+                if (ce == 0) break;                 // no key left (m is the sentinel)
+                if (ce > r) return m;
+                r -= ce;
+                lower = m + 1u;
+            }
+        }
+    } else {
+        int need = top_b - n;                       // theta is the need-th largest key < g
+        uint32_t upper = g;
+        if (need <= kExtract) {
+#pragma unroll 1
+            for (int it = 0; it < kExtract; ++it) {
+                uint32_t m = 0u;
+#pragma unroll
+                for (int j = 0; j < V; ++j) m = valid && k[j] < upper && k[j] > m ? k[j] : m;
+                m = __reduce_max_sync(kFull, m);
+                uint32_t e = 0;
+#pragma unroll
+                for (int j = 0; j < V; ++j) e += valid && k[j] < upper && k[j] == m ? 1u : 0u;
+                const int ce = (int)__reduce_add_sync(kFull, e);
+                if (ce == 0) break;                 // no key below `upper`
+                if (ce >= need) return m;
+                need -= ce;
+                upper = m;
+            }
+        }
+    }
+    return theta_key<V>(k, valid, top_b);
+}
+
 // Slot of this lane holding the element at position B of the total order
 // (score descending, index ascending), or -1: the keys above theta come
 // first, then the keys equal to theta by ascending index V * lane + j.
@@ -152,10 +208,10 @@ __device__ __forceinline__ int theta_slot(const uint32_t (&k)[V], bool valid, ui
         gt += k[j] > th ? 1u : 0u;
         eq += valid && k[j] == th ? 1u : 0u;
     }
-    const int rank = top_b - (int)__reduce_add_sync(kFull, gt);   // 1-based among the equal keys
-    const uint32_t neq = __reduce_add_sync(kFull, eq);
+    const uint32_t both = __reduce_add_sync(kFull, gt | (eq << 16));   // counts <= 256 each
+    const int rank = top_b - (int)(both & 0xffffu);                    // 1-based among the ties
     int before = 0;
-    if (neq > 1u) {                                 // ties at theta: exclusive scan of eq
+    if ((both >> 16) > 1u) {                        // ties at theta: exclusive scan of eq
         uint32_t inc = eq;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -171,51 +227,61 @@ __device__ __forceinline__ int theta_slot(const uint32_t (&k)[V], bool valid, ui
     return slot;
 }
 
-// One coverage term l(s, q): returns the loss, writes g = dl/ds and gq = dl/dq.
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ float rcp_approx(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// One coverage term before its reductions.  With d = s_e - theta_B and
+// u = sigmoid(|d| / tau), v = 1 - u: om_e = 1 - m_e (v if d >= 0, else u) and
+// w_e = q_e m_e (1 - m_e) = q_e u v, so that dl/ds_e = (W [e = e*] - w_e) / tau
+// with W = sum_e w_e (the second part through theta_B = s_{e*}).  Adds the
+// lane's share of l and of W to loss and wsum; the slot of e* comes back.
 template <int V>
-__device__ __forceinline__ float coverage(const float (&s)[V], const float (&q)[V], bool valid,
-                                          int top_b, float inv_tau, int lane, float (&g)[V],
-                                          float (&gq)[V]) {
+__device__ __forceinline__ int coverage(const float (&s)[V], const float (&q)[V], bool valid,
+                                        int top_b, float k2, int lane, uint32_t& guess,
+                                        float (&w)[V], float (&om)[V], float& loss, float& wsum) {
     uint32_t k[V];
 #pragma unroll
     for (int j = 0; j < V; ++j) k[j] = valid ? __float_as_uint(s[j]) : 0u;
-    const uint32_t th = theta_key<V>(k, valid, top_b);
+    const uint32_t th = theta_near<V>(k, valid, top_b, guess);
+    guess = th;
     const int js = theta_slot<V>(k, valid, th, top_b, lane);
     const float theta = __uint_as_float(th);
-    float loss = 0.f, sdm = 0.f;
 #pragma unroll
     for (int j = 0; j < V; ++j) {
-        const float x = (s[j] - theta) * inv_tau;
-        const float E = __expf(-fabsf(x));             // in (0, 1]
-        const float up = __fdividef(1.f, 1.f + E);      // sigmoid(|x|)
-        const float dn = E * up;                        // sigmoid(-|x|)
-        const float om = x >= 0.f ? dn : up;            // 1 - m_e
-        loss = fmaf(q[j], om, loss);
-        const float dm = q[j] * (up * dn) * inv_tau;    // q_e dm_e/ds_e
-        g[j] = -dm;
-        gq[j] = om;
-        sdm += dm;
+        const float d = s[j] - theta;
+        const float E = ex2_approx(-fabsf(d) * k2);     // exp(-|d| / tau), in (0, 1]
+        const float u = rcp_approx(1.f + E);
+        const float v = E * u;
+        om[j] = d >= 0.f ? v : u;
+        loss = fmaf(q[j], om[j], loss);
+        w[j] = q[j] * (u * v);
+        wsum += w[j];
     }
-    loss = warp_sum(loss);
-    sdm = warp_sum(sdm);
-#pragma unroll
-    for (int j = 0; j < V; ++j)
-        if (j == js) g[j] += sdm;                       // through theta_B = s_{e*}
-    return loss;
+    return js;
 }
 
-// Softmax backward of one head row and its store: dz = p (dp - <p, dp>).
-template <int V>
-__device__ __forceinline__ void store_dz(float* row, const float (&p)[V], const float (&d)[V],
-                                         int lane, bool valid) {
-    float dot = 0.f;
-#pragma unroll
-    for (int j = 0; j < V; ++j) dot = fmaf(p[j], d[j], dot);
-    dot = warp_sum(dot);
-    float o[V];
-#pragma unroll
-    for (int j = 0; j < V; ++j) o[j] = p[j] * (d[j] - dot);
-    store_row<V>(row, o, lane, valid);
+// Sums of four per-lane values over the warp in one transposing butterfly
+// (6 shuffles): lanes 0-7 end with the sum of a, 8-15 of b, 16-23 of c,
+// 24-31 of d.
+__device__ __forceinline__ float warp_sum4(float a, float b, float c, float d, int lane) {
+    const bool h16 = (lane & 16) != 0;
+    const float x0 = (h16 ? c : a) + __shfl_xor_sync(kFull, h16 ? a : c, 16);
+    const float x1 = (h16 ? d : b) + __shfl_xor_sync(kFull, h16 ? b : d, 16);
+    const bool h8 = (lane & 8) != 0;
+    float y = (h8 ? x1 : x0) + __shfl_xor_sync(kFull, h8 ? x0 : x1, 8);
+    y += __shfl_xor_sync(kFull, y, 4);
+    y += __shfl_xor_sync(kFull, y, 2);
+    y += __shfl_xor_sync(kFull, y, 1);
+    return y;
 }
 
 template <int V>
@@ -226,8 +292,73 @@ __device__ __forceinline__ void store_zero(float* row, int lane, bool valid) {
     store_row<V>(row, z, lane, valid);
 }
 
+// Softmax backward of up to three head rows and their stores:
+// dz = p (dp - <p, dp>), the three inner products in one butterfly.
+template <int V>
+__device__ __forceinline__ void store_dz3(float* rR, float* rT, float* rS, const float (&pR)[V],
+                                          const float (&dR)[V], const float (&pT)[V],
+                                          const float (&dT)[V], const float (&pS)[V],
+                                          const float (&dS)[V], bool with_s, int lane,
+                                          bool valid) {
+    float a = 0.f, b = 0.f, c = 0.f;
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        a = fmaf(pR[j], dR[j], a);
+        b = fmaf(pT[j], dT[j], b);
+        c = fmaf(pS[j], dS[j], c);
+    }
+    const float y = warp_sum4(a, b, c, 0.f, lane);
+    const float dotR = __shfl_sync(kFull, y, 0);
+    const float dotT = __shfl_sync(kFull, y, 8);
+    const float dotS = __shfl_sync(kFull, y, 16);
+    float o[V];
+#pragma unroll
+    for (int j = 0; j < V; ++j) o[j] = pR[j] * (dR[j] - dotR);
+    store_row<V>(rR, o, lane, valid);
+#pragma unroll
+    for (int j = 0; j < V; ++j) o[j] = pT[j] * (dT[j] - dotT);
+    store_row<V>(rT, o, lane, valid);
+    if (with_s) {
+#pragma unroll
+        for (int j = 0; j < V; ++j) o[j] = pS[j] * (dS[j] - dotS);
+        store_row<V>(rS, o, lane, valid);
+    }
+}
+
+// Both terms of step t of layer l from s^T = p^R_t + p^T_t, p^S_{rho(t+1,l)}
+// and the target q = p^R_{t+1}: their losses (lane 0: l^T, lane 16: l^ST in
+// the returned value), gT = tau dl^T/ds, gST likewise, and the target parts.
+template <int V>
+__device__ __forceinline__ float step_terms(const float (&pR)[V], const float (&pT)[V],
+                                            const float (&pS)[V], const float (&q)[V],
+                                            bool st, bool valid, int top_b, float k2, int lane,
+                                            uint32_t (&guess)[2], float (&wT)[V], float (&omT)[V],
+                                            float (&wST)[V], float (&omST)[V]) {
+    float s[V];
+#pragma unroll
+    for (int j = 0; j < V; ++j) s[j] = __fadd_rn(pR[j], pT[j]);
+    float lT = 0.f, sT = 0.f, lST = 0.f, sST = 0.f;
+    const int jT = coverage<V>(s, q, valid, top_b, k2, lane, guess[0], wT, omT, lT, sT);
+    int jST = -1;
+    if (st) {
+#pragma unroll
+        for (int j = 0; j < V; ++j) s[j] = __fadd_rn(s[j], pS[j]);
+        jST = coverage<V>(s, q, valid, top_b, k2, lane, guess[1], wST, omST, lST, sST);
+    }
+    const float y = warp_sum4(lT, sT, lST, sST, lane);
+    const float WT = __shfl_sync(kFull, y, 8);
+    const float WST = __shfl_sync(kFull, y, 24);
+    // w <- w - W [e = e*], so that dl/ds = -w / tau
+#pragma unroll
+    for (int j = 0; j < V; ++j) {
+        if (j == jT) wT[j] -= WT;
+        if (j == jST) wST[j] -= WST;
+    }
+    return y;
+}
+
 template <int V, bool ALL_VALID>
-__global__ void __launch_bounds__(32 * kLossWarps) cache_loss_kernel(const LossArgs a) {
+__global__ void __launch_bounds__(32 * kLossWarps, V >= 8 ? 2 : 4) cache_loss_kernel(const LossArgs a) {
     const int lane = threadIdx.x & 31;
     const int task = blockIdx.x * kLossWarps + (threadIdx.x >> 5);
     if (task >= a.B * a.L * a.nchunks) return;
@@ -240,106 +371,98 @@ __global__ void __launch_bounds__(32 * kLossWarps) cache_loss_kernel(const LossA
     const bool valid = ALL_VALID || lane < N / V;
     const bool st = a.heads == 3;
     const bool want_grad = a.grad != nullptr;
+    const float k2 = a.k2, cT = a.cT, cST = a.cST, gT = a.gT, gST = a.gST;
     const size_t row3 = (size_t)3 * N;
-    const size_t u_b = (size_t)b * T;
-    auto unit = [&](int t, int ll) { return (u_b + t) * L + ll; };
-    auto prow = [&](int t, int ll, int h) { return a.probs + unit(t, ll) * row3 + (size_t)h * N; };
-    auto grow = [&](int t, int ll, int h) { return a.grad + unit(t, ll) * row3 + (size_t)h * N; };
-    // rho(t + 1, l): (t, L - 1) for l = 0, (t + 1, l - 1) otherwise
-    auto srow = [&](int t) { return l > 0 ? prow(t + 1, l - 1, 2) : prow(t, L - 1, 2); };
-    auto sgrow = [&](int t) { return l > 0 ? grow(t + 1, l - 1, 2) : grow(t, L - 1, 2); };
+    const size_t tok = (size_t)L * row3;                      // one token of one stream
+    // row pointers at token t of unit (b, t, l) (load_row / store_row add the
+    // lane's V elements); p^S of rho(t + 1, l) is (t, L - 1) for l = 0 and
+    // (t + 1, l - 1) otherwise
+    const size_t base = ((size_t)b * T * L + l) * row3;
+    const size_t s_off = l > 0 ? tok + (size_t)2 * N - row3 : (size_t)(L - 1 - l) * row3 + 2 * N;
+    const float* pp = a.probs + base + (size_t)t0 * tok;
+    float* gp = want_grad ? a.grad + base + (size_t)t0 * tok : nullptr;
+    float* lossp = a.loss ? a.loss + (((size_t)b * T + t0) * L + l) * 2 : nullptr;
 
     float pR[V], pT[V], q[V], pS[V], carry[V];
-    float gT[V], gqT[V], gST[V], gqST[V];
+    float wT[V], omT[V], wST[V], omST[V];
 #pragma unroll
     for (int j = 0; j < V; ++j) {
         carry[j] = 0.f;
-        gST[j] = gqST[j] = pS[j] = 0.f;
+        wST[j] = omST[j] = pS[j] = 0.f;
     }
     double sumT = 0.0, sumST = 0.0;
+    uint32_t guess[2] = {0u, 0u};                             // theta^T, theta^ST of the last step
 
     if (t0 > 0) {
         // halo: the two terms of step t0 - 1 give the target part of p^R_{t0}
-        load_row<V>(pR, prow(t0 - 1, l, 0), lane, valid);
-        load_row<V>(pT, prow(t0 - 1, l, 1), lane, valid);
-        load_row<V>(q, prow(t0, l, 0), lane, valid);
-        if (st) load_row<V>(pS, srow(t0 - 1), lane, valid);
-        float s[V];
-#pragma unroll
-        for (int j = 0; j < V; ++j) s[j] = __fadd_rn(pR[j], pT[j]);
-        coverage<V>(s, q, valid, a.top_b, a.inv_tau, lane, gT, gqT);
-        if (st) {
-#pragma unroll
-            for (int j = 0; j < V; ++j) s[j] = __fadd_rn(s[j], pS[j]);
-            coverage<V>(s, q, valid, a.top_b, a.inv_tau, lane, gST, gqST);
-        }
+        const float* hp = pp - tok;
+        load_row<V>(pR, hp, lane, valid);
+        load_row<V>(pT, hp + N, lane, valid);
+        load_row<V>(q, pp, lane, valid);
+        if (st) load_row<V>(pS, hp + s_off, lane, valid);
+        step_terms<V>(pR, pT, pS, q, st, valid, a.top_b, k2, lane, guess, wT, omT, wST, omST);
 #pragma unroll
         for (int j = 0; j < V; ++j) {
-            carry[j] = a.cT * gqT[j] + a.cST * gqST[j];
+            carry[j] = fmaf(cT, omT[j], cST * omST[j]);
             pR[j] = q[j];
         }
     } else {
-        load_row<V>(pR, prow(0, l, 0), lane, valid);
-        if (a.loss && lane == 0) a.loss[unit(0, l) * 2 + 1] = 0.f;     // no l^ST at t = 0
-        if (st && want_grad && l > 0) store_zero<V>(grow(0, l - 1, 2), lane, valid);
+        load_row<V>(pR, pp, lane, valid);
+        if (lossp && lane == 0) lossp[1] = 0.f;                   // no l^ST at t = 0
+        if (st && want_grad && l > 0) store_zero<V>(gp + 2 * N - row3, lane, valid);
     }
 
 #pragma unroll 1
-    for (int t = t0; t < t1; ++t) {
-        load_row<V>(pT, prow(t, l, 1), lane, valid);
-        float dR[V], dT[V];
-        if (t + 1 < T) {
-            load_row<V>(q, prow(t + 1, l, 0), lane, valid);
-            if (st) load_row<V>(pS, srow(t), lane, valid);
-            float s[V];
-#pragma unroll
-            for (int j = 0; j < V; ++j) s[j] = __fadd_rn(pR[j], pT[j]);
-            const float lT = coverage<V>(s, q, valid, a.top_b, a.inv_tau, lane, gT, gqT);
-            float lST = 0.f;
-            if (st) {
-#pragma unroll
-                for (int j = 0; j < V; ++j) s[j] = __fadd_rn(s[j], pS[j]);
-                lST = coverage<V>(s, q, valid, a.top_b, a.inv_tau, lane, gST, gqST);
-            }
-            sumT += (double)lT;
-            sumST += (double)lST;
-            if (a.loss && lane == 0) {
-                a.loss[unit(t, l) * 2 + 0] = lT;
-                a.loss[unit(t + 1, l) * 2 + 1] = st ? lST : 0.f;
+    for (int t = t0; t < t1; ++t, pp += tok) {
+        load_row<V>(pT, pp + N, lane, valid);
+        float dR[V], dT[V], dS[V];
+        const bool next = t + 1 < T;
+        if (next) {
+            load_row<V>(q, pp + tok, lane, valid);
+            if (st) load_row<V>(pS, pp + s_off, lane, valid);
+            const float y = step_terms<V>(pR, pT, pS, q, st, valid, a.top_b, k2, lane, guess, wT,
+                                          omT, wST, omST);
+            if (lane == 0) {
+                sumT += (double)y;
+                if (lossp) lossp[0] = y;
+            } else if (lane == 16) {
+                sumST += (double)y;
+                if (lossp) lossp[(size_t)L * 2 + 1] = st ? y : 0.f;
             }
 #pragma unroll
             for (int j = 0; j < V; ++j) {
-                const float gs = a.cT * gT[j] + a.cST * gST[j];
+                const float gs = -fmaf(gT, wT[j], gST * wST[j]);
                 dT[j] = gs;
                 dR[j] = carry[j] + gs;
-                carry[j] = a.cT * gqT[j] + a.cST * gqST[j];
-            }
-            if (st && want_grad) {
-                float dS[V];
-#pragma unroll
-                for (int j = 0; j < V; ++j) dS[j] = a.cST * gST[j];
-                store_dz<V>(sgrow(t), pS, dS, lane, valid);
+                dS[j] = -gST * wST[j];
+                carry[j] = fmaf(cT, omT[j], cST * omST[j]);
             }
         } else {
             // last token: no l^T here, no l^ST after it
-            if (a.loss && lane == 0) a.loss[unit(t, l) * 2 + 0] = 0.f;
+            if (lossp && lane == 0) lossp[0] = 0.f;
 #pragma unroll
             for (int j = 0; j < V; ++j) {
                 dR[j] = carry[j];
-                dT[j] = 0.f;
+                dT[j] = dS[j] = 0.f;
             }
-            if (st && want_grad && l == 0) store_zero<V>(grow(t, L - 1, 2), lane, valid);
+            if (st && want_grad && l == 0) store_zero<V>(gp + s_off, lane, valid);
         }
         if (want_grad) {
-            store_dz<V>(grow(t, l, 0), pR, dR, lane, valid);
-            store_dz<V>(grow(t, l, 1), pT, dT, lane, valid);
+            store_dz3<V>(gp, gp + N, gp + s_off, pR, dR, pT, dT, pS, dS, st && next, lane,
+                         valid);
+            gp += tok;
         }
+        if (lossp) lossp += (size_t)L * 2;
 #pragma unroll
         for (int j = 0; j < V; ++j) pR[j] = q[j];
     }
-    if (a.partial && lane == 0) {
-        a.partial[(size_t)task * 2 + 0] = sumT;
-        a.partial[(size_t)task * 2 + 1] = sumST;
+    if (a.partial) {
+        sumT = __shfl_sync(kFull, sumT, 0);
+        sumST = __shfl_sync(kFull, sumST, 16);
+        if (lane == 0) {
+            a.partial[(size_t)task * 2 + 0] = sumT;
+            a.partial[(size_t)task * 2 + 1] = sumST;
+        }
     }
 }
 
@@ -386,13 +509,14 @@ int launch_loss_t(const LossArgs& a, cudaStream_t stream) {
 }  // namespace
 
 LossPlan loss_plan(int B, int L, int T) {
-    // About 8192 warp tasks (several waves of resident warps on any current
-    // GPU), chunks of at least 16 tokens so the halo step costs <= 1/16.
+    // About 49152 warp tasks (ten waves of resident warps on a 152-SM GPU,
+    // so the last one idles little), chunks of at least 32 tokens so the halo
+    // step costs <= 1/32.
     LossPlan pl{1, T > 0 ? T : 1};
     if (T <= 0) return pl;
     const long long bl = (long long)B * L;
-    long long n = (8192 + bl - 1) / bl;
-    const long long cap = (T + 15) / 16;
+    long long n = (49152 + bl - 1) / bl;
+    const long long cap = (T + 31) / 32;
     if (n > cap) n = cap;
     if (n < 1) n = 1;
     pl.chunk = (int)((T + n - 1) / n);
@@ -418,9 +542,13 @@ int launch_cache_loss(const crc_problem& p, const float* probs, int T, int heads
     a.top_b = top_b;
     a.chunk = pl.chunk;
     a.nchunks = pl.nchunks;
-    a.inv_tau = (float)(1.0 / tau);
-    a.cT = n_valid > 0 ? (float)(w_T / n_valid) : 0.f;
-    a.cST = n_valid > 0 && heads == 3 ? (float)(w_ST / n_valid) : 0.f;
+    a.k2 = (float)(1.4426950408889634 / tau);
+    const double cT = n_valid > 0 ? w_T / n_valid : 0.0;
+    const double cST = n_valid > 0 && heads == 3 ? w_ST / n_valid : 0.0;
+    a.cT = (float)cT;
+    a.cST = (float)cST;
+    a.gT = (float)(cT / tau);
+    a.gST = (float)(cST / tau);
     int rc;
 #define CRC_LOSS_V(VV)                                                               \
     rc = p.N == 32 * VV ? launch_loss_t<VV, true>(a, stream)                         \

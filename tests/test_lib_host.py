@@ -114,8 +114,8 @@ def test_policy_scan_argument_checks(crc):
 def test_cache_loss_argument_checks(crc):
     lib = crc.load()
     p = crc.problem_of(S.QWEN3_30B)
-    # per-task fp64 sums: B * L tasks per token chunk, 3 chunks of 342 tokens at T = 1024
-    assert crc.crc_loss_workspace_bytes(p, 1024) == (64 * 48 * 3 * 16 + 255) // 256 * 256
+    # per-task fp64 sums: B * L tasks per token chunk, 16 chunks of 64 tokens at T = 1024
+    assert crc.crc_loss_workspace_bytes(p, 1024) == 64 * 48 * 16 * 16
     assert crc.crc_loss_workspace_bytes(p, 0) == 0
     ws = crc.crc_loss_workspace_bytes(p, 8)
     call = lambda T=8, heads=3, top_b=20, tau=0.03, wT=1.0, wST=1.0, probs=256, loss=256, \
