@@ -106,26 +106,34 @@ def workload_config(w, chunk=None):
 
 
 class ClockSampler:
-    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
-    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+    """nvidia-smi samples (every 20 ms) of SM clock, power and throttle reasons
+    during the timed region: the context waits for the first sample before the
+    region starts, and the summary keeps the samples time-stamped inside it."""
+    Q = ("timestamp,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
 
     def __init__(self, gpu_id: str):
         self.gpu_id = gpu_id
         self.proc = None
         self.lines = []
+        self.t0 = self.t1 = None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.Q}",
-                 "--format=csv,noheader,nounits", "-lms", "50"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
+            deadline = time.time() + 5.0
+            while not self.lines and time.time() < deadline and self.proc.poll() is None:
+                time.sleep(0.01)
         except OSError:
             self.proc = None
+        self.t0 = time.time()
         return self
 
     def _read(self):
@@ -133,6 +141,8 @@ class ClockSampler:
             self.lines.append(line.strip())
 
     def __exit__(self, *a):
+        self.t1 = time.time()
+        time.sleep(0.05)
         if self.proc:
             self.proc.terminate()
             try:
@@ -141,25 +151,39 @@ class ClockSampler:
                 self.proc.kill()
             self.t.join(timeout=2)
 
+    @staticmethod
+    def _stamp(text: str):
+        import datetime
+        try:
+            return datetime.datetime.strptime(text.strip(), "%Y/%m/%d %H:%M:%S.%f").timestamp()
+        except ValueError:
+            return None
+
     def summary(self):
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        sm, mx, pw, reasons = [], [], [], set()
         for ln in self.lines:
             parts = [x.strip() for x in ln.split(",")]
-            if len(parts) < 8:
+            if len(parts) < 9:
+                continue
+            ts = self._stamp(parts[0])
+            if ts is None or self.t0 is None or not (self.t0 - 0.03 <= ts <= self.t1 + 0.03):
                 continue
             try:
-                sm.append(float(parts[0]))
-                mx.append(float(parts[1]))
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+                pw.append(float(parts[3]))
             except ValueError:
                 continue
-            for n, v in zip(names, parts[4:8]):
+            for n, v in zip(self.NAMES, parts[5:9]):
                 if v.lower().startswith("active"):
                     reasons.add(n)
         if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0,
+                    "window_s": None if self.t0 is None else round(self.t1 - self.t0, 3)}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
-                "reasons": sorted(reasons), "samples": len(sm)}
+                "sm_min_mhz": min(sm), "power_w": statistics.median(pw),
+                "reasons": sorted(reasons), "samples": len(sm),
+                "window_s": round(self.t1 - self.t0, 3)}
 
 
 def gpu_id_for_smi(torch, dev: int) -> str:
@@ -599,7 +623,9 @@ def main():
 
     # a comparison policy's scan reads p^R only (Spatio-only: and p^S)
     scan_heads = heads if args.policy == "method" else (2 if args.policy == "spatio_lru" else 1)
-    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step, scan_heads)
+    clocks = clk.summary()
+    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step, scan_heads,
+                                         clocks)
     if args.policy != "method" and roof.get("kernel") == "cache_scan_kernel":
         roof["kernel"] = f"cache_scan_policy_kernel ({args.policy})"
 
@@ -626,7 +652,7 @@ def main():
                            workspace_bytes=int(ws_bytes)),
             "roofline": roof, "path_roofline": path_roof, "kernels": kernels,
             "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches),
-            "clocks": clk.summary(),
+            "clocks": clocks,
             "policy": policy_report(P, stats, p, m),
         }
         print(json.dumps(line), flush=True)
@@ -635,10 +661,21 @@ def main():
     return 0
 
 
-def rooflines(kt, w, heads, steps, ms, ms_per_step, scan_heads=None):
+def tensor_peak(pk, clocks):
+    """The bf16 peak that matches the timed region's clock regime: the measured
+    sustained figure (a GEMM held at the power cap) when the SM clock was held
+    by the power cap during the region, else the burst figure."""
+    capped = bool(clocks) and "sw_power_cap" in (clocks.get("reasons") or [])
+    if capped:
+        return pk["bf16_tflops_sustained"], "sustained: sw_power_cap active in the timed region"
+    return pk["bf16_tflops"], "burst"
+
+
+def rooflines(kt, w, heads, steps, ms, ms_per_step, scan_heads=None, clocks=None):
     """Roofline of the dominant kernel (timed live over the timed region) and of
-    the whole path (max of flops at bf16 peak and bytes at HBM bandwidth)."""
+    the whole path (max of flops at the bf16 peak and bytes at HBM bandwidth)."""
     pk, pk_src = peaks()
+    tpk, tpk_kind = tensor_peak(pk, clocks)
     dom = max(("fused", "router", "scan"), key=lambda k: kt[k]["ms"])
     avg_ms = kt[dom]["ms"] / max(1, kt[dom]["launches"])
     t_s = kt[dom]["ms"] / 1000.0
@@ -654,26 +691,28 @@ def rooflines(kt, w, heads, steps, ms, ms_per_step, scan_heads=None):
         flops, bytes_ = algorithmic(w, w.units, heads)
         flops, bytes_ = flops * steps, bytes_ * steps
         kname = f"fused_route_cache_kernel<{w.N},{heads}>"
-    t_flop = flops / (pk["bf16_tflops"] * 1e12)
+    t_flop = flops / (tpk * 1e12)
     t_byte = bytes_ / (pk["hbm_gbs"] * 1e9)
     if t_flop >= t_byte:
-        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": pk["bf16_tflops"],
-                "unit": "TFLOP/s", "frac": t_flop / t_s}
+        roof = {"bound": "tensor", "achieved": flops / t_s / 1e12, "peak": tpk,
+                "unit": "TFLOP/s", "frac": t_flop / t_s,
+                "frac_of_burst": flops / (pk["bf16_tflops"] * 1e12) / t_s,
+                "frac_of_sustained": flops / (pk["bf16_tflops_sustained"] * 1e12) / t_s}
     else:
         roof = {"bound": "hbm", "achieved": bytes_ / t_s / 1e9, "peak": pk["hbm_gbs"],
                 "unit": "GB/s", "frac": t_byte / t_s}
     per_unit, src = committed_traffic(kname, w.name)
     units_per_launch = w.units * steps / max(1, kt[dom]["launches"])
     roof["traffic"] = None if per_unit is None else per_unit * units_per_launch
-    roof.update({"kernel": kname, "peak_source": f"{pk_src} ({'burst' if roof['bound'] == 'tensor' else 'copy'})",
+    roof.update({"kernel": kname, "peak_source": f"{pk_src} ({tpk_kind if roof['bound'] == 'tensor' else 'copy'})",
                  "avg_launch_ms": avg_ms, "launches": kt[dom]["launches"],
                  "share_of_step": kt[dom]["ms"] / ms if ms else None})
     # whole-path roofline (spec definition): max(flops at bf16 peak, bytes at HBM)
     fl, by = algorithmic(w, w.units, heads)
-    t_roof = max(fl / (pk["bf16_tflops"] * 1e12), by / (pk["hbm_gbs"] * 1e9))
+    t_roof = max(fl / (tpk * 1e12), by / (pk["hbm_gbs"] * 1e9))
     path_roof = {"t_roof_ms": 1000 * t_roof, "frac": 1000 * t_roof / ms_per_step,
-                 "bound": "tensor" if fl / (pk["bf16_tflops"] * 1e12) >= by / (pk["hbm_gbs"] * 1e9)
-                 else "hbm"}
+                 "bound": "tensor" if fl / (tpk * 1e12) >= by / (pk["hbm_gbs"] * 1e9)
+                 else "hbm", "tensor_peak": tpk_kind}
     kernels = {k: {"launches": v["launches"], "ms_per_step": v["ms"] / steps}
                for k, v in kt.items() if v["launches"]}
     return roof, path_roof, kernels
@@ -743,7 +782,8 @@ def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
     ms_per_step = ms / args.steps
     units_all = w.units * world
     value = units_all / (ms_per_step / 1000.0)
-    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step)
+    clocks = clk.summary()
+    roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step, None, clocks)
     kernels.pop("synth", None)
     kernels.pop("state", None)
     launches = sum(kt[k]["launches"] for k in ("fused", "router", "scan"))
@@ -764,7 +804,7 @@ def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
             "cpu_baseline": cpu,
             "e2e": None, "e2e_note": "hidden states exceed host and device memory; "
                                      "generated on the device per chunk",
-            "gpu_launches": int(launches), "clocks": clk.summary(),
+            "gpu_launches": int(launches), "clocks": clocks,
             "policy": policy_report(P, stats, p, m),
         }
         print(json.dumps(line), flush=True)

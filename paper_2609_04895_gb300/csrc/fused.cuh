@@ -335,24 +335,41 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
     }
 }
 
-template <int NH, int H>
+// PAIR: the GEMM runs on CTA pairs (tcgen05.mma.cta_group::2, M = 256): each
+// CTA of a pair loads its own 128-row hidden tile and half of the weight rows
+// of every MMA (96 of 192), so a stage carries 37.5 % fewer bytes per flop;
+// the even CTA issues the MMAs into both CTAs' TMEM.
+template <int NH, int H, bool PAIR = false>
 struct FusedCfg {
     using RC = RouterCfg<NH, H>;
     static constexpr int GEMM_WARPS = 6;
     static constexpr int SCAN_WARPS = 10;
     static constexpr int THREADS = 32 * (GEMM_WARPS + SCAN_WARPS);
-    static constexpr int STAGES = imin(8, (232448 - 1024 - 256) / RC::STAGE_BYTES);
-    static constexpr int SMEM_BYTES = 1024 + STAGES * RC::STAGE_BYTES + 256;
+    static constexpr int B_ROWS = PAIR ? RC::NCOL / 2 : RC::NCOL;        // weight rows per CTA
+    static constexpr int B_BOX_ROWS = PAIR ? RC::NCH / 2 : RC::B_BOX_ROWS;
+    static constexpr int B_BOXES = B_ROWS / B_BOX_ROWS;
+    static constexpr int STAGE_BYTES = RC::A_BYTES + B_ROWS * RC::BK * 2;
+    static constexpr uint32_t IDESC = PAIR ? idesc_bf16_f32(2 * RC::BM, RC::NCH) : RC::IDESC;
+    // PAIR: the Temporal head's exps are parked in shared memory (fp32,
+    // [NH/4][128 rows] float4) and p^R's in the spare TMEM columns, so the
+    // accumulator goes back to the MMA after two passes over those heads
+    static constexpr int PARK_T_BYTES = PAIR ? RC::BM * NH * 4 : 0;
+    static constexpr int STAGES = imin(8, (232448 - 1024 - 256 - PARK_T_BYTES) / STAGE_BYTES);
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + PARK_T_BYTES + 256;
     static constexpr int CW = NH < 32 ? NH : 32;     // TMEM columns per load
     static constexpr int NCHK = NH / CW;
     static_assert(STAGES >= 2, "pipeline depth");
+    static_assert(!PAIR || (RC::NMMA == 2 && RC::NACC == 1 && B_BOXES == RC::NMMA),
+                  "CTA pairs: two MMAs per K step, one accumulator");
+    static_assert((STAGE_BYTES % 1024) == 0 && ((B_BOX_ROWS * 128) % 1024) == 0,
+                  "swizzle atom alignment");
 };
 
-template <int NH, int H, int V, bool ALL_VALID, int KP>
+template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR = false>
 __global__ void __launch_bounds__(512, 1)
     fused_route_cache_kernel(const __grid_constant__ CUtensorMap tmap_h,
                              const __grid_constant__ CUtensorMap tmap_w, FusedArgs a) {
-    using Cfg = FusedCfg<NH, H>;
+    using Cfg = FusedCfg<NH, H, PAIR>;
     using RC = typename Cfg::RC;
     using RL = RingLayout<NH>;
     constexpr int CW = Cfg::CW;
@@ -374,7 +391,9 @@ __global__ void __launch_bounds__(512, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* tiles = smem;
-    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * RC::STAGE_BYTES);
+    float4* tpark = reinterpret_cast<float4*>(smem + Cfg::STAGES * Cfg::STAGE_BYTES);
+    uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem + Cfg::STAGES * Cfg::STAGE_BYTES +
+                                                     Cfg::PARK_T_BYTES);
     uint64_t* empty_bar = full_bar + Cfg::STAGES;
     uint64_t* tfull_bar = empty_bar + Cfg::STAGES;
     uint64_t* tempty_bar = tfull_bar + RC::NACC;
@@ -383,6 +402,12 @@ __global__ void __launch_bounds__(512, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
+    // PAIR: rank 0 issues the MMAs for both CTAs; the tile loops below step by
+    // gridDim.x from blockIdx.x, so the two CTAs of a pair hold the adjacent
+    // tiles 2j and 2j + 1 (same token block and layer: the launch makes the
+    // stream count even) at every iteration.
+    const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+    const bool leader = rank == 0u;
 
     StateHeader* hdr = reinterpret_cast<StateHeader*>(a.state);
     uint32_t* err = &hdr->error;
@@ -400,7 +425,7 @@ __global__ void __launch_bounds__(512, 1)
         }
         for (int s = 0; s < RC::NACC; ++s) {
             mbar_init(&tfull_bar[s], 1);
-            mbar_init(&tempty_bar[s], 4);
+            mbar_init(&tempty_bar[s], PAIR ? 8 : 4);       // both CTAs' epilogue warps
         }
         mbar_init(drain_bar, 1);
         fence_mbar_init();
@@ -408,11 +433,17 @@ __global__ void __launch_bounds__(512, 1)
         tma_prefetch_desc(&tmap_w);
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, RC::TMEM_COLS);
-        tmem_relinquish();
+        if constexpr (PAIR) {
+            tmem_alloc_pair(tmem_slot, RC::TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(tmem_slot, RC::TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
+    if constexpr (PAIR) cluster_sync();             // the peer's barriers exist before any remote use
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     const int num_tiles = hdr_ok ? a.num_tiles : 0;
@@ -424,12 +455,17 @@ __global__ void __launch_bounds__(512, 1)
             const uint64_t pol_w = l2_evict_last_policy();
             int stage = 0, issued = 0, failed = 0;
             uint32_t phase = 0;
+            // PAIR: both CTAs' loads of a stage complete on the even CTA's full
+            // barrier, which expects the bytes of both
+            const uint32_t lead_full = PAIR ? cluster_map(&full_bar[0], 0u) : 0u;
             for (int k = blockIdx.x; k < num_tiles && !failed; k += gridDim.x) {
                 const int tb = k / a.tiles_per_tb;
                 const int rem = k % a.tiles_per_tb;
                 const int l = rem / a.n_bg, bg = rem % a.n_bg;
                 for (int kb = 0; kb < a.kblocks; ++kb) {
-                    if (!mbar_wait(&empty_bar[stage], phase ^ 1) || ld_acquire_u32(abort_flag)) {
+                    const bool freed = PAIR ? mbar_wait_cluster(&empty_bar[stage], phase ^ 1)
+                                            : mbar_wait(&empty_bar[stage], phase ^ 1);
+                    if (!freed || ld_acquire_u32(abort_flag)) {
                         if (!ld_acquire_u32(abort_flag)) {
                             latch_error(err, CRC_ETIMEOUT);
                             atomicExch(abort_flag, 1u);
@@ -437,15 +473,28 @@ __global__ void __launch_bounds__(512, 1)
                         failed = 1;
                         break;
                     }
-                    uint8_t* sa = tiles + stage * RC::STAGE_BYTES;
+                    uint8_t* sa = tiles + stage * Cfg::STAGE_BYTES;
                     uint8_t* sw = sa + RC::A_BYTES;
-                    mbar_arrive_expect_tx(&full_bar[stage], RC::STAGE_BYTES);
-                    tma_load_4d(sa, &tmap_h, &full_bar[stage], kb * RC::BK, l, tb * a.TB,
-                                bg * a.SB, pol_h);
+                    if constexpr (PAIR) {
+                        if (leader) mbar_arrive_expect_tx(&full_bar[stage], 2 * Cfg::STAGE_BYTES);
+                        const uint32_t fb = lead_full + (uint32_t)(stage * 8);
+                        tma_load_4d_pair(sa, &tmap_h, fb, kb * RC::BK, l, tb * a.TB, bg * a.SB,
+                                         pol_h);
+                        // rows [c*NCH + rank*NCH/2, +NCH/2) of MMA c's weight block
 #pragma unroll
-                    for (int c = 0; c < RC::B_BOXES; ++c)
-                        tma_load_3d(sw + c * RC::B_BOX_ROWS * 128, &tmap_w, &full_bar[stage],
-                                    kb * RC::BK, c * RC::B_BOX_ROWS, l, pol_w);
+                        for (int c = 0; c < Cfg::B_BOXES; ++c)
+                            tma_load_3d_pair(sw + c * Cfg::B_BOX_ROWS * 128, &tmap_w, fb,
+                                             kb * RC::BK, c * RC::NCH + (int)rank * Cfg::B_BOX_ROWS,
+                                             l, pol_w);
+                    } else {
+                        mbar_arrive_expect_tx(&full_bar[stage], Cfg::STAGE_BYTES);
+                        tma_load_4d(sa, &tmap_h, &full_bar[stage], kb * RC::BK, l, tb * a.TB,
+                                    bg * a.SB, pol_h);
+#pragma unroll
+                        for (int c = 0; c < Cfg::B_BOXES; ++c)
+                            tma_load_3d(sw + c * Cfg::B_BOX_ROWS * 128, &tmap_w, &full_bar[stage],
+                                        kb * RC::BK, c * Cfg::B_BOX_ROWS, l, pol_w);
+                    }
                     ++issued;
                     if (++stage == Cfg::STAGES) {
                         stage = 0;
@@ -455,7 +504,9 @@ __global__ void __launch_bounds__(512, 1)
             }
             int s = stage;
             uint32_t ph = phase;
-            for (int k = 0; k < imin(issued, Cfg::STAGES); ++k) {
+            // (PAIR: only the even CTA's barriers see the loads; the odd CTA
+            // stays until its loads landed through the final cluster barrier)
+            for (int k = 0; k < ((PAIR && !leader) ? 0 : imin(issued, Cfg::STAGES)); ++k) {
                 if (--s < 0) {
                     s = Cfg::STAGES - 1;
                     ph ^= 1;
@@ -463,13 +514,17 @@ __global__ void __launch_bounds__(512, 1)
                 if (!mbar_wait(&full_bar[s], ph)) latch_error(err, CRC_ETIMEOUT);
             }
         }
+    } else if (warp == 1 && PAIR && !leader) {
+        // the odd CTA's MMA warp only takes part in the TMEM allocation
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA
         if (lane == 0) {
             int stage = 0, acc = 0, failed = 0;
             uint32_t phase = 0, acc_phase = 0;
             for (int k = blockIdx.x; k < num_tiles && !failed; k += gridDim.x) {
-                if (!mbar_wait(&tempty_bar[acc], acc_phase ^ 1)) {
+                const bool acc_free = PAIR ? mbar_wait_cluster(&tempty_bar[acc], acc_phase ^ 1)
+                                           : mbar_wait(&tempty_bar[acc], acc_phase ^ 1);
+                if (!acc_free) {
                     latch_error(err, CRC_ETIMEOUT);
                     atomicExch(abort_flag, 1u);
                     break;
@@ -477,14 +532,16 @@ __global__ void __launch_bounds__(512, 1)
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(acc * RC::ACC_COLS);
                 for (int kb = 0; kb < a.kblocks; ++kb) {
-                    if (!mbar_wait(&full_bar[stage], phase)) {
+                    const bool landed = PAIR ? mbar_wait_cluster(&full_bar[stage], phase)
+                                             : mbar_wait(&full_bar[stage], phase);
+                    if (!landed) {
                         latch_error(err, CRC_ETIMEOUT);
                         atomicExch(abort_flag, 1u);
                         failed = 1;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t sa = smem_u32(tiles + stage * RC::STAGE_BYTES);
+                    const uint32_t sa = smem_u32(tiles + stage * Cfg::STAGE_BYTES);
                     const uint32_t sw = sa + RC::A_BYTES;
 #pragma unroll
                     for (int kk = 0; kk < RC::BK / 16; ++kk) {
@@ -492,19 +549,29 @@ __global__ void __launch_bounds__(512, 1)
 #pragma unroll
                         for (int c = 0; c < RC::NMMA; ++c) {
                             const uint64_t bdesc =
-                                sw128_kmajor_desc(sw + c * RC::NCH * 128 + kk * 32);
-                            umma_bf16(d_tmem + c * RC::NCH, adesc, bdesc, RC::IDESC,
-                                      (kb | kk) != 0);
+                                sw128_kmajor_desc(sw + c * Cfg::B_BOX_ROWS * 128 + kk * 32);
+                            if constexpr (PAIR)
+                                umma_bf16_pair(d_tmem + c * RC::NCH, adesc, bdesc, Cfg::IDESC,
+                                               (kb | kk) != 0);
+                            else
+                                umma_bf16(d_tmem + c * RC::NCH, adesc, bdesc, Cfg::IDESC,
+                                          (kb | kk) != 0);
                         }
                     }
-                    umma_commit(&empty_bar[stage]);
+                    if constexpr (PAIR)
+                        umma_commit_pair(&empty_bar[stage]);
+                    else
+                        umma_commit(&empty_bar[stage]);
                     if (++stage == Cfg::STAGES) {
                         stage = 0;
                         phase ^= 1;
                     }
                 }
                 if (failed) break;
-                umma_commit(&tfull_bar[acc]);
+                if constexpr (PAIR)
+                    umma_commit_pair(&tfull_bar[acc]);
+                else
+                    umma_commit(&tfull_bar[acc]);
                 if (RC::NACC == 2) {
                     acc ^= 1;
                     if (acc == 0) acc_phase ^= 1;
@@ -512,7 +579,10 @@ __global__ void __launch_bounds__(512, 1)
                     acc_phase ^= 1;
                 }
             }
-            umma_commit(drain_bar);
+            if constexpr (PAIR)
+                umma_commit_pair_local(drain_bar);
+            else
+                umma_commit(drain_bar);
             if (!mbar_wait(drain_bar, 0)) latch_error(err, CRC_ETIMEOUT);
         }
     } else if (warp < Cfg::GEMM_WARPS) {
@@ -522,8 +592,21 @@ __global__ void __launch_bounds__(512, 1)
         const uint32_t target_per_tile = 3u * (uint32_t)a.SB;
         int acc = 0;
         uint32_t acc_phase = 0;
+        // PAIR: the accumulator is released to the even CTA's MMA issuer
+        const uint32_t tempty_peer = PAIR ? cluster_map(&tempty_bar[0], 0u) : 0u;
+        auto release_acc = [&](int which) {
+            if constexpr (PAIR) {
+                if (!leader) {
+                    mbar_arrive_remote(tempty_peer + (uint32_t)(which * 8));
+                    return;
+                }
+            }
+            mbar_arrive(&tempty_bar[which]);
+        };
         for (int k = blockIdx.x; k < num_tiles; k += gridDim.x) {
-            if (!mbar_wait(&tfull_bar[acc], acc_phase)) {
+            const bool filled = PAIR ? mbar_wait_cluster(&tfull_bar[acc], acc_phase)
+                                     : mbar_wait(&tfull_bar[acc], acc_phase);
+            if (!filled) {
                 latch_error(err, CRC_ETIMEOUT);
                 atomicExch(abort_flag, 1u);
                 break;
@@ -555,7 +638,6 @@ __global__ void __launch_bounds__(512, 1)
                     tmem_cols<CW>(tbase + (uint32_t)(2 * NH + c * CW), z);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
-#pragma unroll
                     m = max_of<CW>(z, m);
                 }
                 // each exp(z - max) is computed once and parked in the
@@ -605,6 +687,12 @@ __global__ void __launch_bounds__(512, 1)
             r1.init(mR);
             t0.init(mT);
             t1.init(mT);
+            // With a single accumulator, p^R is parked in the spare TMEM columns
+            // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
+            // before the Top-K selection runs (PAIR: already its exps, with the
+            // Temporal exps in shared memory, before s^T is formed).
+            constexpr bool PARK = RC::NACC == 1 && RC::NCOL + NH <= RC::ACC_COLS;
+            const uint32_t pbase = tbase + (uint32_t)RC::NCOL;
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
                 tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
@@ -614,20 +702,53 @@ __global__ void __launch_bounds__(512, 1)
                 pin_cols<CW>(y);
                 chunk_exp(c, z, r0, r1);
                 chunk_exp(c, y, t0, t1);
-                tmem_put<CW>(tbase + (uint32_t)(c * CW), z);
-                tmem_put<CW>(tbase + (uint32_t)(NH + c * CW), y);
+                if constexpr (PAIR) {
+                    tmem_put<CW>(pbase + (uint32_t)(c * CW), z);
+#pragma unroll
+                    for (int q = 0; q < CW / 4; ++q)
+                        tpark[(c * CW / 4 + q) * 128 + row] =
+                            make_float4(y[4 * q], y[4 * q + 1], y[4 * q + 2], y[4 * q + 3]);
+                } else {
+                    tmem_put<CW>(tbase + (uint32_t)(c * CW), z);
+                    tmem_put<CW>(tbase + (uint32_t)(NH + c * CW), y);
+                }
             }
             tmem_st_wait();
             const float rR = head_inv(r0.part(), r1.part()), rT = head_inv(t0.part(), t1.part());
-            // With a single accumulator, p^R is parked in the spare TMEM columns
-            // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
-            // before the Top-K selection runs.
-            constexpr bool PARK = RC::NACC == 1 && RC::NCOL + NH <= RC::ACC_COLS;
-            const uint32_t pbase = tbase + (uint32_t)RC::NCOL;
             TopKAcc<KP> topk;
             topk.init();
+            if constexpr (PAIR) {
+                tc_fence_before();                        // accumulator columns fully read
+                __syncwarp();
+                if (lane == 0) release_acc(acc);
 #pragma unroll 1
-            for (int c = 0; c < NCHK; ++c) {
+                for (int c = 0; c < NCHK; ++c) {
+                    tmem_cols<CW>(pbase + (uint32_t)(c * CW), z);
+#pragma unroll
+                    for (int q = 0; q < CW / 4; ++q) {
+                        const float4 f = tpark[(c * CW / 4 + q) * 128 + row];
+                        y[4 * q] = f.x;
+                        y[4 * q + 1] = f.y;
+                        y[4 * q + 2] = f.z;
+                        y[4 * q + 3] = f.w;
+                    }
+                    tmem_ld_wait();
+                    pin_cols<CW>(z);
+                    retention_in_place<CW>(z, y, rR, rT);         // z = p^R, y = s^T
+                    if (ok) {
+#pragma unroll
+                        for (int q = 0; q < CW / 4; ++q)
+                            sT_p[(size_t)(c * CW / 4 + q) * 128 + row] =
+                                make_float4(y[4 * q], y[4 * q + 1], y[4 * q + 2], y[4 * q + 3]);
+                    }
+                    tmem_put<CW>(pbase + (uint32_t)(c * CW), z);
+#pragma unroll
+                    for (int g = 0; g < CW; g += 16) topk.add16(z + g);
+                }
+                tmem_st_wait();
+            }
+#pragma unroll 1
+            for (int c = 0; c < (PAIR ? 0 : NCHK); ++c) {
                 tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
                 tmem_cols<CW>(tbase + (uint32_t)(NH + c * CW), y);
                 tmem_ld_wait();
@@ -647,11 +768,11 @@ __global__ void __launch_bounds__(512, 1)
                     for (int g = 0; g < CW; g += 16) topk.add16(z + g);
                 }
             }
-            if constexpr (PARK) {
+            if constexpr (PARK && !PAIR) {
                 tmem_st_wait();
                 tc_fence_before();                        // accumulator columns fully read
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+                if (lane == 0) release_acc(acc);
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(pbase + (uint32_t)(c * CW), z);
@@ -677,7 +798,7 @@ __global__ void __launch_bounds__(512, 1)
                     if (c == NCHK - 1) {                  // accumulator fully read
                         tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+                        if (lane == 0) release_acc(acc);
                     }
                     scale_in_place<CW>(z, rR);                    // p^R
                 }
@@ -724,9 +845,15 @@ __global__ void __launch_bounds__(512, 1)
     }
     tc_fence_before();
     __syncthreads();
+    // PAIR: neither CTA leaves (or frees TMEM) while the other may still
+    // arrive on its barriers or have MMAs write its TMEM
+    if constexpr (PAIR) cluster_sync();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem_base, RC::TMEM_COLS);
+        if constexpr (PAIR)
+            tmem_dealloc_pair(tmem_base, RC::TMEM_COLS);
+        else
+            tmem_dealloc(tmem_base, RC::TMEM_COLS);
     }
     // the last CTA to finish advances the token counter and flips the carry slot
     if (threadIdx.x == 0) {

@@ -42,28 +42,62 @@ inline FusedPlan fused_plan(const crc_problem& p, int T) {
     return f;
 }
 
-template <int NH, int H, int V, bool ALL_VALID, int KP>
+// PAIR launches clusters of two CTAs (the GEMM on CTA pairs), cooperatively so
+// that every CTA is resident; a device that refuses that launch gets the
+// single-CTA kernel from then on (CRC_EUNSUPPORTED).
+template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR = false>
 int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                    void* state, void* workspace, cudaStream_t stream) {
-    using Cfg = FusedCfg<NH, H>;
+    using Cfg = FusedCfg<NH, H, PAIR>;
     using RC = typename Cfg::RC;
     const FusedPlan f = fused_plan(p, T);
+    if (PAIR && (f.SB != 1 || f.n_bg % 2 != 0)) return CRC_EUNSUPPORTED;
+    auto kern = fused_route_cache_kernel<NH, H, V, ALL_VALID, KP, PAIR>;
+    // -1: not set up yet in this process; 0: refused; else the grid
+    static int grid = -1;
+    if (grid == 0) return CRC_EUNSUPPORTED;
+    if (grid < 0) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 Cfg::SMEM_BYTES) != cudaSuccess) {
+            (void)cudaGetLastError();
+            grid = 0;
+            return CRC_EUNSUPPORTED;
+        }
+        if (PAIR) {
+            cudaLaunchAttribute at[1];
+            at[0].id = cudaLaunchAttributeClusterDimension;
+            at[0].val.clusterDim.x = 2;
+            at[0].val.clusterDim.y = 1;
+            at[0].val.clusterDim.z = 1;
+            cudaLaunchConfig_t c = {};
+            c.gridDim = dim3((unsigned)(sm_count() / 2 * 2));
+            c.blockDim = dim3(Cfg::THREADS);
+            c.dynamicSmemBytes = Cfg::SMEM_BYTES;
+            c.attrs = at;
+            c.numAttrs = 1;
+            int ncl = 0;
+            if (cudaOccupancyMaxActiveClusters(&ncl, (const void*)kern, &c) != cudaSuccess ||
+                ncl < 1) {
+                (void)cudaGetLastError();
+                grid = 0;
+                return CRC_EUNSUPPORTED;
+            }
+            grid = std::min(2 * ncl, sm_count() / 2 * 2);
+        } else {
+            int per_sm = 0;
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Cfg::THREADS,
+                                                              Cfg::SMEM_BYTES) != cudaSuccess ||
+                per_sm < 1) {
+                (void)cudaGetLastError();
+                grid = 0;
+                return CRC_EUNSUPPORTED;
+            }
+            grid = sm_count();
+        }
+    }
     CUtensorMap mh, mw;
     if (!make_hidden_map(&mh, hidden, p.B, T, p.L, p.d, f.TB, f.SB)) return CRC_ECUDA;
-    if (!make_weight_map(&mw, w_cat, p.L, 3 * NH, p.d, RC::B_BOX_ROWS)) return CRC_ECUDA;
-    auto kern = fused_route_cache_kernel<NH, H, V, ALL_VALID, KP>;
-    static bool attr_set = false;
-    if (!attr_set) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 Cfg::SMEM_BYTES) != cudaSuccess)
-            return CRC_ECUDA;
-        attr_set = true;
-    }
-    int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Cfg::THREADS,
-                                                      Cfg::SMEM_BYTES) != cudaSuccess ||
-        per_sm < 1)
-        return CRC_EUNSUPPORTED;
+    if (!make_weight_map(&mw, w_cat, p.L, 3 * NH, p.d, Cfg::B_BOX_ROWS)) return CRC_ECUDA;
     uint8_t* ws = static_cast<uint8_t*>(workspace);
     if (cudaMemsetAsync(ws, 0, f.ctl_bytes, stream) != cudaSuccess) return CRC_ECUDA;
     FusedArgs a;
@@ -91,9 +125,32 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
     a.ring_base = ws + f.ctl_bytes;
     a.slot_bytes = f.slot_bytes;
     void* args[] = {(void*)&mh, (void*)&mw, (void*)&a};
-    const int grid = sm_count();
     cudaError_t e;
-    {
+    if (PAIR) {
+        cudaLaunchAttribute at[2];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = 2;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        at[1].id = cudaLaunchAttributeCooperative;
+        at[1].val.cooperative = 1;
+        cudaLaunchConfig_t c = {};
+        c.gridDim = dim3((unsigned)grid);
+        c.blockDim = dim3(Cfg::THREADS);
+        c.dynamicSmemBytes = Cfg::SMEM_BYTES;
+        c.stream = stream;
+        c.attrs = at;
+        c.numAttrs = 2;
+        {
+            ProfScope prof(CRC_KERNEL_FUSED, stream);
+            e = cudaLaunchKernelExC(&c, (const void*)kern, args);
+        }
+        if (e != cudaSuccess) {
+            (void)cudaGetLastError();
+            grid = 0;
+            return CRC_EUNSUPPORTED;
+        }
+    } else {
         ProfScope prof(CRC_KERNEL_FUSED, stream);
         e = cudaLaunchCooperativeKernel((const void*)kern, grid, Cfg::THREADS, args,
                                         Cfg::SMEM_BYTES, stream);
@@ -118,6 +175,20 @@ int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint1
                                                        stream);                               \
     return CRC_EUNSUPPORTED;
     if (p.R > 0) {
+        if constexpr (NH == 128) {
+            // the GEMM on CTA pairs when the tiles pair up, else one CTA per tile
+            int rc = CRC_EUNSUPPORTED;
+            if (p.K <= 2)
+                rc = launch_fused_t<NH, 3, V, ALL_VALID, 2, true>(p, hidden, w_cat, T, state,
+                                                                 workspace, stream);
+            else if (p.K <= 4)
+                rc = launch_fused_t<NH, 3, V, ALL_VALID, 4, true>(p, hidden, w_cat, T, state,
+                                                                 workspace, stream);
+            else if (p.K <= 8)
+                rc = launch_fused_t<NH, 3, V, ALL_VALID, 8, true>(p, hidden, w_cat, T, state,
+                                                                 workspace, stream);
+            if (rc != CRC_EUNSUPPORTED) return rc;
+        }
         CRC_FUSED_KP(3)
     } else {
         CRC_FUSED_KP(2)
