@@ -663,9 +663,12 @@ def main():
 
 def tensor_peak(pk, clocks):
     """The bf16 peak that matches the timed region's clock regime: the measured
-    sustained figure (a GEMM held at the power cap) when the SM clock was held
-    by the power cap during the region, else the burst figure."""
-    capped = bool(clocks) and "sw_power_cap" in (clocks.get("reasons") or [])
+    sustained figure (a GEMM held at the power cap) when the power cap held the
+    SM clock for most of the region (median below 95 % of the maximum), else
+    the burst figure."""
+    capped = (bool(clocks) and "sw_power_cap" in (clocks.get("reasons") or [])
+              and clocks.get("sm_mhz") is not None
+              and clocks["sm_mhz"] < 0.95 * (clocks.get("sm_max_mhz") or clocks["sm_mhz"]))
     if capped:
         return pk["bf16_tflops_sustained"], "sustained: sw_power_cap active in the timed region"
     return pk["bf16_tflops"], "burst"
