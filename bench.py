@@ -54,11 +54,13 @@ def parse_args():
                     help="proactive-load bound R (default: the workload's; the large shape takes 2 or 8)")
     ap.add_argument("--tokens", type=int, default=0,
                     help="override T (a smaller case, e.g. for an ncu capture)")
-    ap.add_argument("--only", choices=["fused", "pair", "router", "scan", "loss"], default="fused",
+    ap.add_argument("--only", choices=["fused", "pair", "router", "scan", "loss", "transfer"],
+                    default="fused",
                     help="fused: crc_route_and_cache as one fused kernel (default); pair: "
                          "crc_route_scores then crc_cache_scan; router / scan: one part alone; "
                          "loss: the soft Top-B coverage losses and their gradient "
-                         "(crc_cache_loss) on the router's probabilities")
+                         "(crc_cache_loss) on the router's probabilities; transfer: one "
+                         "stream's expert copies (crc_transfer_plan / crc_transfer_replay)")
     ap.add_argument("--top-b", type=int, default=0,
                     help="with --only loss: B of the soft Top-B loss (0 = the paper's: 20 for "
                          "N = 128, 8 for N = 32)")
@@ -483,6 +485,101 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
     return 0
 
 
+TRANSFER_METRIC = "expert bytes moved per second (host pool -> HBM cache slots)"
+
+
+def run_transfer(args, P, C, w, p, dev, stream, rank, world):
+    """Replays the expert copies of stream 0: the router and the scan run once
+    with cache traces (untimed), crc_transfer_plan turns the stream's cache
+    sets into copies, and each timed step enqueues all of them
+    (crc_transfer_replay, one cudaMemcpyAsync of expert_bytes per copy) from a
+    pinned host pool to a device cache of L x C slots.  The pool holds 64
+    expert images, copy (l, e) reading image (l N + e) mod 64: the bytes and
+    sizes are the real ones, the images repeat."""
+    import numpy as np
+    import torch
+    T = args.tokens or 256
+    w = w.with_(T=T)
+    Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
+    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
+                           rho_l=w.rho_l, device=dev)
+    st = P.State(p, device=dev)
+    tr = P.Trace.alloc(p, w.T, device=dev, caches=True)
+    P.route_and_cache(p, hd, Wd, st, tr)
+    stats = st.read(want_chain_counters=True)
+    assert stats["error"] == 0, stats
+    del hd, Wd
+    mid = tr.cache_mid[0].cpu().numpy()
+    aft = tr.cache_after[0].cpu().numpy()
+    t0 = time.perf_counter()
+    plan, _ = P.transfer_plan(p, mid, aft)
+    plan_ms = 1000 * (time.perf_counter() - t0)
+    eb = int(p.expert_bytes)
+    counters = stats["chain_counters"].reshape(w.B, w.L, 3)[0]
+    assert len(plan) == int(counters[:, 1].sum() + counters[:, 2].sum())
+    pool_n = 64
+    pool = torch.empty(pool_n * eb, dtype=torch.uint8, pin_memory=True)
+    pool.fill_(7)
+    slots = torch.empty((w.L, w.C, eb), dtype=torch.uint8, device=dev)
+    # the host link's copy rate: one pinned copy of the whole pool, best of 3
+    big = slots.view(-1)[:pool.numel()]
+    best = None
+    for _ in range(3):
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        big.copy_(pool, non_blocking=True)
+        a1.record(stream)
+        torch.cuda.synchronize()
+        ms = a0.elapsed_time(a1)
+        best = ms if best is None else min(best, ms)
+    peak_gbs = pool.numel() / (best / 1000.0) / 1e9
+
+    def step():
+        C.crc_transfer_replay(p, plan.ctypes.data, len(plan), pool.data_ptr(), pool_n,
+                              slots.data_ptr(), stream)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    steps = args.steps
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(gpu_id_for_smi(torch, dev.index or 0)) as clk:
+        e0.record(stream)
+        for _ in range(steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    ms_per_step = ms / steps
+    moved = len(plan) * eb
+    value = moved / (ms_per_step / 1000.0)
+    m = P.metrics({k: stats[k] for k in stats}, p)
+    tok_ms = ms_per_step / T
+    if rank == 0:
+        line = {
+            "metric": TRANSFER_METRIC, "value": value, "unit": "B/s", "n_gpus": world,
+            "steps": steps, "warmup": max(3, args.warmup), "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "u8",
+            "data": "synthetic",
+            "config": dict(workload_config(w), path="transfer", stream=0,
+                           copies_per_step=int(len(plan)), bytes_per_step=int(moved),
+                           proactive_copies=int((plan["proactive"] == 1).sum()),
+                           pool_images=pool_n, plan_ms=plan_ms),
+            "roofline": {"bound": "c2c", "achieved": value / 1e9, "peak": peak_gbs,
+                         "unit": "GB/s", "frac": value / 1e9 / peak_gbs, "traffic": None,
+                         "kernel": "cudaMemcpyAsync host -> device (one per planned copy)",
+                         "peak_source": "one pinned host -> device copy of the whole pool, "
+                                        "measured in this run"},
+            "transfer_ms_per_token": tok_ms,
+            "load_model": {"hit": m["hit"], "adj_hit": m["adj_hit"],
+                           "load_MB_per_token": m["load_per_token_bytes"] / 1e6},
+            "cpu_baseline": None, "e2e": None, "gpu_launches": 0,
+            "clocks": clk.summary(),
+        }
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -552,6 +649,8 @@ def main():
     stream = torch.cuda.current_stream()
     if args.only == "loss":
         return run_loss(args, P, C, w, p, dev, stream, rank, world)
+    if args.only == "transfer":
+        return run_transfer(args, P, C, w, p, dev, stream, rank, world)
     if 2 * w.B * w.T * w.L * w.d > STREAM_BYTES:
         return run_streamed(args, P, C, w, p, heads, dev, stream, rank, world)
 

@@ -72,11 +72,16 @@ typedef struct crc_problem {
 } crc_problem;
 
 /* Optional per-access trace of one call, device pointers, each may be NULL.
- * T is the call's token count and t the token index within the call. */
+ * T is the call's token count and t the token index within the call.  The
+ * cache sets are bitmasks of NW = ceil(N / 32) words per access (expert e is
+ * bit e % 32 of word e / 32); they are written by the method's scan only
+ * (crc_cache_scan, crc_route_and_cache), not by the comparison policies. */
 typedef struct crc_trace {
     uint8_t *topk_dev;       /* [B][T][L][K] native Top-K, rank order          */
     uint8_t *misses_dev;     /* [B][T][L] demand misses |S \ C~|               */
     uint8_t *proactive_dev;  /* [B][T][L] proactive loads of the refinement    */
+    uint32_t *cache_mid_dev; /* [B][T][L][NW] cache after Algorithm 2 (C~)     */
+    uint32_t *cache_after_dev; /* [B][T][L][NW] cache after UpdateCache      */
 } crc_trace;
 
 /* Totals over all streams and layers since crc_state_init (Sec. 4.1). */
@@ -271,6 +276,49 @@ int crc_cache_loss(const crc_problem *p, const float *probs_dev, int32_t T, int3
                    int32_t top_b, double tau, double w_T, double w_ST, float *loss_dev,
                    double *means_dev, float *grad_dev, void *workspace_dev,
                    size_t workspace_bytes, void *stream);
+
+/* Expert transfers (the expert pool of Sec. 2 and the transfers counted in
+ * Sec. 4.1): the cache simulation's load decisions for one stream as copies
+ * of expert weights from a host pool into a device cache of C slots per
+ * layer.  One planned copy: */
+typedef struct crc_transfer {
+    int32_t t;          /* token of the access (index into the trace)          */
+    int32_t l;          /* layer                                               */
+    int32_t expert;     /* expert loaded                                       */
+    int32_t slot;       /* destination slot, 0 .. C-1 of layer l               */
+    int32_t evicted;    /* expert that left that slot in this phase, -1 if free */
+    int32_t proactive;  /* 1: Algorithm 2 proactive load; 0: demand load       */
+} crc_transfer;
+
+/* Host-only planning from one stream's cache trace (crc_trace's cache_mid and
+ * cache_after of that stream, host copies, [T][L][NW] each).  Per access, the
+ * experts that entered the cache in the refinement phase (C~ \ C) are the
+ * proactive loads and those that entered in UpdateCache (C+ \ C~) the demand
+ * loads, so the plan holds exactly P + D copies; an expert that leaves frees
+ * its slot.  Slots: within a phase the freed slots are taken first (ascending
+ * slot), by the loaded experts in ascending expert order, then free slots.
+ *   start_host   [L][NW] cache before token 0, checked against slot_expert
+ *                (NULL: not checked);
+ *   slot_expert  [L][C] in: the expert in each slot before token 0 (-1 free);
+ *                out: after the last token;
+ *   out          room for max_out copies, or NULL to count only;
+ *                *n_out receives the number of copies.
+ * CRC_EINVAL on bad sizes, inconsistent masks (more than C members, an
+ * expert in two slots) or more copies than max_out (with out given). */
+int crc_transfer_plan(const crc_problem *p, int32_t T, const uint32_t *mid_host,
+                      const uint32_t *after_host, const uint32_t *start_host,
+                      int32_t *slot_expert, crc_transfer *out, int64_t max_out,
+                      int64_t *n_out);
+
+/* Enqueues the planned copies on `stream`, in plan order, one
+ * cudaMemcpyAsync of expert_bytes each: from pool_host (pinned host memory,
+ * pool_experts expert images; copy (l, e) reads image (l * N + e) %
+ * pool_experts, so a pool of L * N images holds every expert once) to
+ * slots_dev [L][C][expert_bytes].  Asynchronous; CRC_ECUDA if a copy cannot
+ * be enqueued. */
+int crc_transfer_replay(const crc_problem *p, const crc_transfer *plan, int64_t n,
+                        const void *pool_host, int64_t pool_experts, void *slots_dev,
+                        void *stream);
 
 /* Synchronises the device and returns (then clears) the error latched by
  * calls without a state (crc_route_scores), CRC_OK if none. */

@@ -29,7 +29,18 @@ class crc_problem(ctypes.Structure):
 
 class crc_trace(ctypes.Structure):
     _fields_ = [("topk_dev", ctypes.c_void_p), ("misses_dev", ctypes.c_void_p),
-                ("proactive_dev", ctypes.c_void_p)]
+                ("proactive_dev", ctypes.c_void_p), ("cache_mid_dev", ctypes.c_void_p),
+                ("cache_after_dev", ctypes.c_void_p)]
+
+
+class crc_transfer(ctypes.Structure):
+    _fields_ = [("t", ctypes.c_int32), ("l", ctypes.c_int32), ("expert", ctypes.c_int32),
+                ("slot", ctypes.c_int32), ("evicted", ctypes.c_int32),
+                ("proactive", ctypes.c_int32)]
+
+
+TRANSFER_DTYPE = np.dtype([("t", np.int32), ("l", np.int32), ("expert", np.int32),
+                           ("slot", np.int32), ("evicted", np.int32), ("proactive", np.int32)])
 
 
 class crc_stats(ctypes.Structure):
@@ -77,6 +88,8 @@ EXPORTS = [
      [PP, P, I32, P, SZ, ctypes.POINTER(crc_trace), I32, I32, P]),
     ("crc_state_read_aux", ctypes.c_int, [PP, P, SZ, P, P]),
     ("crc_loss_workspace_bytes", SZ, [PP, I32]),
+    ("crc_transfer_plan", ctypes.c_int, [PP, I32, P, P, P, P, P, ctypes.c_int64, P]),
+    ("crc_transfer_replay", ctypes.c_int, [PP, P, ctypes.c_int64, P, ctypes.c_int64, P, P]),
     ("crc_cache_loss", ctypes.c_int, [PP, P, I32, I32, I32, D, D, D, P, P, P, P, SZ, P]),
     ("crc_launch_count", U64, []),
     ("crc_strerror", ctypes.c_char_p, [ctypes.c_int]),
@@ -207,6 +220,21 @@ def crc_cache_loss(p: crc_problem, probs_ptr: int, T: int, heads: int, top_b: in
         "crc_cache_loss")
 
 
+def crc_transfer_plan(p: crc_problem, T: int, mid_ptr, after_ptr, start_ptr, slot_expert_ptr,
+                      out_ptr, max_out: int) -> int:
+    n = ctypes.c_int64(0)
+    _ck(load().crc_transfer_plan(ctypes.byref(p), T, mid_ptr, after_ptr, start_ptr,
+                                 slot_expert_ptr, out_ptr, max_out, ctypes.byref(n)),
+        "crc_transfer_plan")
+    return int(n.value)
+
+
+def crc_transfer_replay(p: crc_problem, plan_ptr, n: int, pool_ptr, pool_experts: int,
+                        slots_ptr, stream=None):
+    _ck(load().crc_transfer_replay(ctypes.byref(p), plan_ptr, n, pool_ptr, pool_experts,
+                                   slots_ptr, _stream(stream)), "crc_transfer_replay")
+
+
 def crc_workspace_bytes(p: crc_problem, chunk_tokens: int) -> int:
     return int(load().crc_workspace_bytes(ctypes.byref(p), chunk_tokens))
 
@@ -311,16 +339,52 @@ class Trace:
     topk: object
     misses: object
     proactive: object
+    cache_mid: object = None
+    cache_after: object = None
 
     @staticmethod
-    def alloc(p: crc_problem, T: int, device="cuda") -> "Trace":
+    def alloc(p: crc_problem, T: int, device="cuda", caches: bool = False) -> "Trace":
+        """caches: also the cache sets after the refinement and after the update
+        ([B][T][L][NW] uint32 bitmasks)."""
         import torch
+        nw = (p.N + 31) // 32
+        mk = (lambda: torch.zeros((p.B, T, p.L, nw), dtype=torch.int32, device=device)) \
+            if caches else (lambda: None)
         return Trace(torch.zeros((p.B, T, p.L, p.K), dtype=torch.uint8, device=device),
                      torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device),
-                     torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device))
+                     torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device), mk(), mk())
 
     def c(self) -> crc_trace:
-        return crc_trace(_ptr(self.topk), _ptr(self.misses), _ptr(self.proactive))
+        return crc_trace(_ptr(self.topk), _ptr(self.misses), _ptr(self.proactive),
+                         _ptr(self.cache_mid), _ptr(self.cache_after))
+
+
+def transfer_plan(p: crc_problem, cache_mid, cache_after, slot_expert=None, start=None):
+    """crc_transfer_plan for one stream: cache_mid / cache_after [T][L][NW]
+    (host arrays, uint32 bit patterns).  Returns (plan, slot_expert after the
+    last token); plan is a structured array of TRANSFER_DTYPE."""
+    mid = np.ascontiguousarray(cache_mid).view(np.uint32)
+    aft = np.ascontiguousarray(cache_after).view(np.uint32)
+    T = mid.shape[0]
+    se = (np.full((p.L, p.C), -1, np.int32) if slot_expert is None
+          else np.ascontiguousarray(slot_expert, dtype=np.int32).copy())
+    st = None if start is None else np.ascontiguousarray(start).view(np.uint32)
+    args = (mid.ctypes.data, aft.ctypes.data, None if st is None else st.ctypes.data)
+    scratch = se.copy()                      # the counting pass moves a copy of the map
+    n = crc_transfer_plan(p, T, *args, scratch.ctypes.data, None, 0)
+    plan = np.zeros(n, TRANSFER_DTYPE)
+    crc_transfer_plan(p, T, *args, se.ctypes.data, plan.ctypes.data if n else None, n)
+    return plan, se
+
+
+def transfer_replay(p: crc_problem, plan, pool, slots, pool_experts=None, stream=None):
+    """crc_transfer_replay: pool a pinned host tensor of pool_experts expert
+    images (default: all of it), slots a device tensor [L][C][expert_bytes]."""
+    plan = np.ascontiguousarray(plan, dtype=TRANSFER_DTYPE)
+    nbytes = pool.numel() * pool.element_size()
+    pe = pool_experts or nbytes // int(p.expert_bytes)
+    crc_transfer_replay(p, plan.ctypes.data if len(plan) else None, len(plan), pool.data_ptr(),
+                        pe, slots.data_ptr(), stream)
 
 
 def route_scores(p: crc_problem, hidden, w_cat, heads: int = 3, out=None, stream=None):

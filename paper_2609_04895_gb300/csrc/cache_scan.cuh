@@ -30,6 +30,8 @@ struct ScanArgs {
     uint8_t* trace_topk;     // [B][T][L][K] or null
     uint8_t* trace_miss;     // [B][T][L] or null
     uint8_t* trace_pro;      // [B][T][L] or null
+    uint32_t* trace_mid;     // [B][T][L][NW] cache after the refinement, or null
+    uint32_t* trace_after;   // [B][T][L][NW] cache after UpdateCache, or null
     int trace_T, trace_t0;   // trace arrays span trace_T tokens; this call starts at trace_t0
     int B, T, L, N, K, C, R;
 };
@@ -393,6 +395,18 @@ __device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V]
     return pro;
 }
 
+// This lane's cache bits as the chain's NW bitmask words at dst.
+template <int V>
+__device__ __forceinline__ void store_cache_words(uint32_t cache, int lane, int N, uint32_t* dst) {
+    const int NW = (N + 31) >> 5;
+    const int e0 = lane * V;
+    for (int w = 0; w < NW; ++w) {
+        const uint32_t contrib = (e0 < N && (e0 >> 5) == w) ? (cache << (e0 & 31)) : 0u;
+        const uint32_t word = __reduce_or_sync(kFull, contrib);
+        if (lane == 0) dst[w] = word;
+    }
+}
+
 // One access at (t, l) from the three router probabilities: s^T, the native
 // Top-K (given as a set, or popped in rank order when the trace wants the
 // order), then scan_apply.  Writes the trace.
@@ -402,7 +416,8 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
                                           bool refine, uint32_t valid, int lane, int K, int C,
                                           int R, bool have_sel, uint32_t sel_in,
                                           uint8_t* topk_out, uint8_t* miss_out,
-                                          uint8_t* pro_out) {
+                                          uint8_t* pro_out, uint32_t* mid_out = nullptr,
+                                          uint32_t* after_out = nullptr, int N = 0) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
     float sT[V];
 #pragma unroll
@@ -430,8 +445,17 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
             }
         }
     }
-    int nD;
-    const int pro = scan_apply<V, ALL_VALID>(cr, sT, pS, refine, valid, lane, K, C, R, sel, &nD);
+    int nD, pro;
+    if (mid_out) {
+        // the refinement on its own, so the cache between the two phases is seen
+        pro = refine ? scan_refine<V, ALL_VALID>(cr, pS, valid, lane, C, R) : 0;
+        store_cache_words<V>(cr.cache, lane, N, mid_out);
+        scan_apply<V, ALL_VALID>(cr, sT, pS, false, valid, lane, K, C, R, sel, &nD);
+        cr.pro += (uint32_t)pro;
+    } else {
+        pro = scan_apply<V, ALL_VALID>(cr, sT, pS, refine, valid, lane, K, C, R, sel, &nD);
+    }
+    if (after_out) store_cache_words<V>(cr.cache, lane, N, after_out);
     if (want_topk && lane < K) topk_out[lane] = (uint8_t)my_topk;
     if (lane == 0) {
         if (miss_out) *miss_out = (uint8_t)nD;
@@ -533,7 +557,10 @@ __global__ void __launch_bounds__(128) cache_scan_kernel(ScanArgs a) {
             scan_step<V, ALL_VALID>(cr, cR.v, cT.v, cS.v, want_s && (t0 + t >= 1), valid, lane, a.K, a.C,
                          a.R, batch_sel, sel_in, a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
                          a.trace_miss ? a.trace_miss + unit : nullptr,
-                         a.trace_pro ? a.trace_pro + unit : nullptr);
+                         a.trace_pro ? a.trace_pro + unit : nullptr,
+                         a.trace_mid ? a.trace_mid + unit * (size_t)((N + 31) >> 5) : nullptr,
+                         a.trace_after ? a.trace_after + unit * (size_t)((N + 31) >> 5) : nullptr,
+                         N);
             cR = nR;
             cT = nT;
             cS = nS;
