@@ -353,14 +353,14 @@ struct FusedCfg {
     // PAIR: the Temporal head's exps are parked in shared memory (fp32,
     // [NH/4][128 rows] float4) and p^R's in the spare TMEM columns, so the
     // accumulator goes back to the MMA after two passes over those heads
-    static constexpr int PARK_T_BYTES = PAIR ? RC::BM * NH * 4 : 0;
+    static constexpr bool PARK_T = PAIR && RC::NACC == 1;
+    static constexpr int PARK_T_BYTES = PARK_T ? RC::BM * NH * 4 : 0;
     static constexpr int STAGES = imin(8, (232448 - 1024 - 256 - PARK_T_BYTES) / STAGE_BYTES);
     static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + PARK_T_BYTES + 256;
     static constexpr int CW = NH < 32 ? NH : 32;     // TMEM columns per load
     static constexpr int NCHK = NH / CW;
     static_assert(STAGES >= 2, "pipeline depth");
-    static_assert(!PAIR || (RC::NMMA == 2 && RC::NACC == 1 && B_BOXES == RC::NMMA),
-                  "CTA pairs: two MMAs per K step, one accumulator");
+    static_assert(!PAIR || B_BOXES == RC::NMMA, "CTA pairs: one weight box per MMA half");
     static_assert((STAGE_BYTES % 1024) == 0 && ((B_BOX_ROWS * 128) % 1024) == 0,
                   "swizzle atom alignment");
 };
@@ -702,7 +702,7 @@ __global__ void __launch_bounds__(512, 1)
                 pin_cols<CW>(y);
                 chunk_exp(c, z, r0, r1);
                 chunk_exp(c, y, t0, t1);
-                if constexpr (PAIR) {
+                if constexpr (Cfg::PARK_T) {
                     tmem_put<CW>(pbase + (uint32_t)(c * CW), z);
 #pragma unroll
                     for (int q = 0; q < CW / 4; ++q)
@@ -717,7 +717,7 @@ __global__ void __launch_bounds__(512, 1)
             const float rR = head_inv(r0.part(), r1.part()), rT = head_inv(t0.part(), t1.part());
             TopKAcc<KP> topk;
             topk.init();
-            if constexpr (PAIR) {
+            if constexpr (Cfg::PARK_T) {
                 tc_fence_before();                        // accumulator columns fully read
                 __syncwarp();
                 if (lane == 0) release_acc(acc);
@@ -748,7 +748,7 @@ __global__ void __launch_bounds__(512, 1)
                 tmem_st_wait();
             }
 #pragma unroll 1
-            for (int c = 0; c < (PAIR ? 0 : NCHK); ++c) {
+            for (int c = 0; c < (Cfg::PARK_T ? 0 : NCHK); ++c) {
                 tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
                 tmem_cols<CW>(tbase + (uint32_t)(NH + c * CW), y);
                 tmem_ld_wait();
@@ -768,7 +768,7 @@ __global__ void __launch_bounds__(512, 1)
                     for (int g = 0; g < CW; g += 16) topk.add16(z + g);
                 }
             }
-            if constexpr (PARK && !PAIR) {
+            if constexpr (PARK && !Cfg::PARK_T) {
                 tmem_st_wait();
                 tc_fence_before();                        // accumulator columns fully read
                 __syncwarp();

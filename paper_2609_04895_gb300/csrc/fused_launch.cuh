@@ -159,11 +159,37 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
     return e == cudaSuccess ? CRC_OK : CRC_ECUDA;
 }
 
+// The GEMM on CTA pairs (N = 128: three heads, or two in update-only mode)
+// when the tiles pair up; CRC_EUNSUPPORTED sends the call to one CTA per tile.
+template <int NH, int H, int V, bool ALL_VALID>
+int launch_fused_pair(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
+                      void* state, void* workspace, cudaStream_t stream) {
+    if constexpr (NH != 128) {
+        return CRC_EUNSUPPORTED;
+    } else {
+        if (p.K <= 2)
+            return launch_fused_t<NH, H, V, ALL_VALID, 2, true>(p, hidden, w_cat, T, state,
+                                                                workspace, stream);
+        if (p.K <= 4)
+            return launch_fused_t<NH, H, V, ALL_VALID, 4, true>(p, hidden, w_cat, T, state,
+                                                                workspace, stream);
+        if (p.K <= 8)
+            return launch_fused_t<NH, H, V, ALL_VALID, 8, true>(p, hidden, w_cat, T, state,
+                                                                workspace, stream);
+        return CRC_EUNSUPPORTED;
+    }
+}
+
 // Dispatch on heads (R > 0 needs the Spatio head) and the Top-K network width.
 template <int NH, int V, bool ALL_VALID>
 int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat,
                        int T, void* state, void* workspace, cudaStream_t stream) {
 #define CRC_FUSED_KP(HV)                                                                      \
+    {                                                                                         \
+        const int rc = launch_fused_pair<NH, HV, V, ALL_VALID>(p, hidden, w_cat, T, state,    \
+                                                               workspace, stream);            \
+        if (rc != CRC_EUNSUPPORTED) return rc;                                                \
+    }                                                                                         \
     if (p.K <= 2)                                                                             \
         return launch_fused_t<NH, HV, V, ALL_VALID, 2>(p, hidden, w_cat, T, state, workspace, \
                                                        stream);                               \
@@ -175,20 +201,6 @@ int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint1
                                                        stream);                               \
     return CRC_EUNSUPPORTED;
     if (p.R > 0) {
-        if constexpr (NH == 128) {
-            // the GEMM on CTA pairs when the tiles pair up, else one CTA per tile
-            int rc = CRC_EUNSUPPORTED;
-            if (p.K <= 2)
-                rc = launch_fused_t<NH, 3, V, ALL_VALID, 2, true>(p, hidden, w_cat, T, state,
-                                                                 workspace, stream);
-            else if (p.K <= 4)
-                rc = launch_fused_t<NH, 3, V, ALL_VALID, 4, true>(p, hidden, w_cat, T, state,
-                                                                 workspace, stream);
-            else if (p.K <= 8)
-                rc = launch_fused_t<NH, 3, V, ALL_VALID, 8, true>(p, hidden, w_cat, T, state,
-                                                                 workspace, stream);
-            if (rc != CRC_EUNSUPPORTED) return rc;
-        }
         CRC_FUSED_KP(3)
     } else {
         CRC_FUSED_KP(2)
