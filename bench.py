@@ -809,7 +809,7 @@ def rooflines(kt, w, heads, steps, ms, ms_per_step, scan_heads=None, clocks=None
     roof.update({"kernel": kname, "peak_source": f"{pk_src} ({tpk_kind if roof['bound'] == 'tensor' else 'copy'})",
                  "avg_launch_ms": avg_ms, "launches": kt[dom]["launches"],
                  "share_of_step": kt[dom]["ms"] / ms if ms else None})
-    # whole-path roofline (spec definition): max(flops at bf16 peak, bytes at HBM)
+    # whole-path roofline: the slower of the flops at the bf16 peak and the bytes at HBM bandwidth
     fl, by = algorithmic(w, w.units, heads)
     t_roof = max(fl / (tpk * 1e12), by / (pk["hbm_gbs"] * 1e9))
     path_roof = {"t_roof_ms": 1000 * t_roof, "frac": 1000 * t_roof / ms_per_step,
