@@ -352,6 +352,11 @@ FUSED_CASES = [
     ("r0", S.QWEN3_30B.with_(B=40, T=19, L=4, R=0, C=16)),          # 2 heads, partial group
     ("n64-one-layer", S.TINY.with_(N=64, K=3, C=9, R=5, B=6, T=50, L=1, d=192)),
     ("k1", S.TINY.with_(K=1, C=2, R=2, B=9, T=33)),
+    # 128-token tiles of one stream: N = 128 runs on CTA pairs when B is even
+    ("pairs-ragged", S.QWEN3_30B.with_(B=4, T=300, L=3, d=256)),     # blocks of 100 | 128, 72
+    ("pairs-r0", S.QWEN3_30B.with_(B=6, T=260, L=2, R=0, C=16, d=256)),
+    ("pairs-k4", S.QWEN3_30B.with_(B=2, T=256, L=2, K=4, C=12, R=3, d=192)),
+    ("odd-b-one-cta", S.QWEN3_30B.with_(B=5, T=200, L=3, d=256)),
 ]
 
 
