@@ -197,7 +197,10 @@ size_t crc_fused_workspace_bytes(const crc_problem *p);
  * hidden_dev bf16 [B][T][L][d]; w_cat_dev bf16 [L][3N][d] (the S head is
  * not computed when R = 0).  The router scores never leave the workspace.
  * With workspace_bytes >= crc_fused_workspace_bytes(p) (and no trace, K <= 8)
- * the call is one fused kernel; otherwise workspace_dev holds the scores of one
+ * the call is one fused kernel; for N = 128 with 128-token tiles of one stream
+ * (T > 64) and an even stream count its GEMM runs on CTA pairs (clusters of
+ * two, tcgen05 cta_group::2), otherwise one CTA per tile, with the same
+ * results.  Without that workspace, workspace_dev holds the scores of one
  * chunk of tokens, the chunk length being the largest that fits (at least one
  * token must fit, see crc_workspace_bytes).  256-byte alignment for the
  * workspace. */
