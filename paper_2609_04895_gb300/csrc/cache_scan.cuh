@@ -472,7 +472,7 @@ __device__ __forceinline__ uint32_t lane_bits(const uint32_t* words, int lane, i
 }
 
 template <int V, bool ALL_VALID, int KP>
-__global__ void __launch_bounds__(128) cache_scan_kernel(ScanArgs a) {
+__global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArgs a) {
     // Top-K sets of the next 32 tokens of each warp's chain, one row per token
     __shared__ uint32_t sel_s[4][32][8];
     StateHeader* hdr = reinterpret_cast<StateHeader*>(a.state);
