@@ -85,6 +85,30 @@ def peaks():
         return dict(FALLBACK_PEAKS), "fallback"
 
 
+def rank_seed(rank: int) -> int:
+    """Seed of a rank's synthetic hidden states: under torchrun every rank runs
+    its own B streams (weak scaling), so no two ranks replay the same data."""
+    return 1000 * rank
+
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The slowest rank's time: the job ends when the last rank does
+    (all_reduce MAX on the rank's device; one process: x itself)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank: int, world: int, ms_per_step: float) -> float:
+    """Whole-job throughput: the units every rank processed over the slowest
+    rank's time per step."""
+    return units_per_rank * world / (ms_per_step / 1000.0)
+
+
 def algorithmic(w, units: int, heads: int):
     """Algorithmic flops and HBM bytes of the fused step for `units` decisions:
     2*d*H*N flops per unit; bf16 hidden state read once (2d bytes), the
@@ -380,7 +404,7 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
     import torch.distributed as dist
     top_b, tau = loss_settings(args, w)
     Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
-    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
+    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=rank_seed(rank), rho_t=w.rho_t,
                            rho_l=w.rho_l, device=dev)
     probs = P.route_scores(p, hd, Wd, heads=3)
     del hd, Wd
@@ -412,14 +436,11 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
         torch.cuda.synchronize()
         launches = C.crc_launch_count() - n0
         kt = C.crc_profile_end()
-    ms = e0.elapsed_time(e1)
+    ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
         dist.barrier()
     ms_per_step = ms / args.steps
-    value = w.units * world / (ms_per_step / 1000.0)
+    value = job_rate(w.units, world, ms_per_step)
     L_T, L_ST = (float(x) for x in means.cpu())
 
     # roofline of the loss kernel: probabilities read once, gradient and losses written once
@@ -456,12 +477,8 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
             out.copy_(means, non_blocking=True)
         f1.record(stream)
         torch.cuda.synchronize()
-        ems = f0.elapsed_time(f1)
-        if world > 1:
-            t = torch.tensor([ems], device=dev)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
-        e2e = {"value": w.units * world / (ems / args.steps / 1000.0), "unit": LOSS_UNIT,
+        ems = max_over_ranks(f0.elapsed_time(f1), world, dev)
+        e2e = {"value": job_rate(w.units, world, ems / args.steps), "unit": LOSS_UNIT,
                "h2d_bytes_per_step": int(probs.numel() * 4), "d2h_bytes_per_step": 16,
                "ms_per_step": ems / args.steps}
         del host
@@ -501,7 +518,7 @@ def run_transfer(args, P, C, w, p, dev, stream, rank, world):
     T = args.tokens or 256
     w = w.with_(T=T)
     Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
-    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
+    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=rank_seed(rank), rho_t=w.rho_t,
                            rho_l=w.rho_l, device=dev)
     st = P.State(p, device=dev)
     tr = P.Trace.alloc(p, w.T, device=dev, caches=True)
@@ -656,7 +673,7 @@ def main():
 
     # inputs, resident in HBM before timing (untimed generation)
     Wd = P.synth_weights(w.L, w.N, w.d, seed=0, device=dev)
-    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t,
+    hd, _ = P.synth_hidden(w.B, w.T, w.L, w.d, seed=rank_seed(rank), rho_t=w.rho_t,
                            rho_l=w.rho_l, device=dev)
     chunk = args.chunk or w.T
     ws_bytes = (C.crc_fused_workspace_bytes(p) if args.only == "fused" and not args.chunk
@@ -710,15 +727,12 @@ def main():
         torch.cuda.synchronize()
         launches = C.crc_launch_count() - n0
         kt = C.crc_profile_end()
-    ms = e0.elapsed_time(e1)
+    ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
         dist.barrier()
     ms_per_step = ms / args.steps
     units_all = w.units * world
-    value = units_all / (ms_per_step / 1000.0)
+    value = job_rate(w.units, world, ms_per_step)
 
     # a comparison policy's scan reads p^R only (Spatio-only: and p^S)
     scan_heads = heads if args.policy == "method" else (2 if args.policy == "spatio_lru" else 1)
@@ -850,7 +864,7 @@ def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
             t0 = c * CH
             n = min(CH, w.T - t0)
             h = hflat[: w.B * n * w.L * w.d].view(w.B, n, w.L, w.d)
-            P.synth_hidden(w.B, n, w.L, w.d, seed=1000 * rank, rho_t=w.rho_t, rho_l=w.rho_l,
+            P.synth_hidden(w.B, n, w.L, w.d, seed=rank_seed(rank), rho_t=w.rho_t, rho_l=w.rho_l,
                            t0=t0, carry=carry, out=h, device=dev)
             if timed:
                 evs[c][0].record(stream)
@@ -877,13 +891,10 @@ def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
             ms += step(True)
         kt = C.crc_profile_end()
     stats = st.read()
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world, dev)
     ms_per_step = ms / args.steps
     units_all = w.units * world
-    value = units_all / (ms_per_step / 1000.0)
+    value = job_rate(w.units, world, ms_per_step)
     clocks = clk.summary()
     roof, path_roof, kernels = rooflines(kt, w, heads, args.steps, ms, ms_per_step, None, clocks)
     kernels.pop("synth", None)
@@ -942,11 +953,7 @@ def end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all
     t0 = time.perf_counter()
     for _ in range(args.steps):
         r = e2e_step()
-    dt = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([dt], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        dt = float(t.item())
+    dt = max_over_ranks(time.perf_counter() - t0, world, dev)
     assert r["error"] == 0
     return {"value": units_all * args.steps / dt, "unit": UNIT,
             "h2d_bytes_per_step": int(h_host.numel() * h_host.element_size()),
