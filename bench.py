@@ -834,6 +834,7 @@ def rooflines(kt, w, heads, steps, ms, ms_per_step, scan_heads=None, clocks=None
     return roof, path_roof, kernels
 
 
+E2E_CHUNK = 128          # tokens per host-to-device copy of the end-to-end step
 STREAM_BYTES = 128 << 30     # hidden states above this are generated per chunk
 STREAM_CHUNK = 128           # tokens per chunk of a streamed workload
 
@@ -927,23 +928,26 @@ def run_streamed(args, P, C, w, p, heads, dev, stream, rank, world):
 
 
 def end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all):
-    """The same metric through the C ABI with the step's inputs copied from
-    pinned host memory and its counters read back, inside the timed region."""
+    """The same metric through the C ABI's host-input call: every step copies
+    its hidden states from pinned host memory (crc_host_alloc's huge pages; in
+    128-token chunks, each copy overlapping the step on the previous chunk) and
+    reads its counters back, inside the timed region."""
     import torch
     import torch.distributed as dist
     hd = held.pop()
-    h_host = torch.empty(hd.shape, dtype=hd.dtype, pin_memory=True)
+    h_host = P.pinned_empty(hd.shape, hd.dtype)
     h_host.copy_(hd)
     del hd
     torch.cuda.empty_cache()
-    h_dev = torch.empty(h_host.shape, dtype=h_host.dtype, device=dev)
+    chunk = min(E2E_CHUNK, w.T)
+    staging = torch.empty(C.crc_host_staging_bytes(p, chunk), dtype=torch.uint8, device=dev)
     torch.cuda.synchronize()
 
     def e2e_step():
-        h_dev.copy_(h_host, non_blocking=True)
         st.init()
-        C.crc_route_and_cache(p, h_dev.data_ptr(), Wd.data_ptr(), w.T, st.ptr, st.nbytes,
-                              None, ws.data_ptr(), ws.numel(), stream)
+        C.crc_route_and_cache_host(p, h_host.data_ptr(), Wd.data_ptr(), w.T, chunk, st.ptr,
+                                   st.nbytes, staging.data_ptr(), staging.numel(),
+                                   ws.data_ptr(), ws.numel(), stream)
         return st.read()      # synchronises; reads the step's counters back
 
     for _ in range(2):
@@ -955,10 +959,32 @@ def end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all
         r = e2e_step()
     dt = max_over_ranks(time.perf_counter() - t0, world, dev)
     assert r["error"] == 0
+    h2d = int(h_host.numel() * h_host.element_size())
     return {"value": units_all * args.steps / dt, "unit": UNIT,
-            "h2d_bytes_per_step": int(h_host.numel() * h_host.element_size()),
+            "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": int(256 + p.B * p.L * 64),
-            "ms_per_step": 1000 * dt / args.steps}
+            "ms_per_step": 1000 * dt / args.steps,
+            "call": f"crc_route_and_cache_host, {chunk}-token chunks",
+            "host_link_gbs": host_link_gbs(h_host, staging, stream),
+            "h2d_gbs": h2d / (dt / args.steps) / 1e9}
+
+
+def host_link_gbs(h_host, dev_buf, stream) -> float:
+    """This run's host-to-device copy rate: one plain pinned copy of up to
+    4 GiB (best of 3, CUDA events), the ceiling for the end-to-end step."""
+    import torch
+    n = min(h_host.numel() * h_host.element_size(), dev_buf.numel(), 4 << 30)
+    src = h_host.view(-1).view(torch.uint8)[:n]
+    dst = dev_buf[:n]
+    best = float("inf")
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        dst.copy_(src, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        best = min(best, e0.elapsed_time(e1) / 1e3)
+    return n / best / 1e9
 
 
 if __name__ == "__main__":

@@ -55,7 +55,8 @@ enum {
     CRC_ETIMEOUT = 4,      /* a bounded device wait ran out (latched)         */
     CRC_ESTATE = 5,        /* state buffer too small, uninitialised or made
                               for another problem (latched when seen on GPU)  */
-    CRC_EDEVICE = 6        /* other device-side failure (latched)             */
+    CRC_EDEVICE = 6,       /* other device-side failure (latched)             */
+    CRC_ENOMEM = 7         /* host memory could not be mapped                 */
 };
 
 /* The problem statement (Sec. 2): sizes and budgets.  One per state. */
@@ -208,6 +209,51 @@ int crc_route_and_cache(const crc_problem *p, const uint16_t *hidden_dev,
                         const uint16_t *w_cat_dev, int32_t T, void *state_dev,
                         size_t state_bytes, const crc_trace *trace,
                         void *workspace_dev, size_t workspace_bytes, void *stream);
+
+/* Device bytes of the two staging halves crc_route_and_cache_host uses for
+ * chunks of `chunk_tokens` tokens: 2 x B x chunk_tokens x L x d bf16, each
+ * half rounded up to 256 bytes.  0 if p is invalid or chunk_tokens < 1. */
+size_t crc_host_staging_bytes(const crc_problem *p, int32_t chunk_tokens);
+
+/* Pinned (page-locked, CUDA-registered) host memory for the host-input call:
+ * an anonymous mapping aligned to the kernel's transparent huge-page size,
+ * advised MADV_HUGEPAGE and faulted in before registration, so that a
+ * multi-GB buffer is covered by few large pages (copies of a 12.9 GB buffer
+ * in cudaHostAlloc's small pages ran at 40-60 GB/s about one time in three,
+ * against a steady 210 GB/s from huge pages).  *out receives the pointer
+ * (huge-page aligned, at least `bytes` long); CRC_ENOMEM if the mapping fails,
+ * CRC_ECUDA if registration fails (nothing is left allocated).  Free with
+ * crc_host_free only; crc_host_free(NULL) is a no-op and a pointer this
+ * library did not hand out gives CRC_EINVAL. */
+int crc_host_alloc(size_t bytes, void **out);
+int crc_host_free(void *ptr);
+
+/* crc_route_and_cache with the hidden states in HOST memory (no counterpart
+ * in the paper: the copy from the host is the serving system's, Sec. 2).
+ *   hidden_host   bf16 [B][T][L][d] in host memory, 16-byte aligned; pinned
+ *                 (page-locked, e.g. from crc_host_alloc) memory lets the
+ *                 copies overlap the compute; pageable memory gives the same
+ *                 results without overlap
+ *   chunk_tokens  tokens per copy; the call moves tokens [t0, t0 + chunk) of
+ *                 every stream into one staging half (a 2-D copy on a copy
+ *                 stream the call creates and destroys) while `stream` runs
+ *                 the step on the previous chunk in the other half
+ *   staging_dev   device buffer of crc_host_staging_bytes(p, min(chunk, T))
+ *                 bytes, 256-byte aligned
+ * workspace_dev / workspace_bytes as in crc_route_and_cache (with
+ * crc_fused_workspace_bytes every chunk is one fused kernel); no trace.
+ * Results are bit-identical to crc_route_and_cache over all T tokens (the
+ * calls on successive chunks continue the same state).  The call returns
+ * once everything is queued; all of its work, copies included, is ordered
+ * before later work on `stream`, so neither the host buffer nor the staging
+ * buffer may be reused before `stream` has passed the call.  On an error
+ * part of the work may have been queued: synchronise `stream` before
+ * freeing the buffers. */
+int crc_route_and_cache_host(const crc_problem *p, const uint16_t *hidden_host,
+                             const uint16_t *w_cat_dev, int32_t T, int32_t chunk_tokens,
+                             void *state_dev, size_t state_bytes, void *staging_dev,
+                             size_t staging_bytes, void *workspace_dev, size_t workspace_bytes,
+                             void *stream);
 
 /* ------------------------------------------------------------------------ */
 /* Allocation-free variant (no counterpart in the paper)                    */

@@ -8,6 +8,7 @@ raised.
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import threading
 from dataclasses import dataclass
@@ -17,7 +18,8 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libcrc.so")
 
-CRC_OK, CRC_EINVAL, CRC_EUNSUPPORTED, CRC_ECUDA, CRC_ETIMEOUT, CRC_ESTATE, CRC_EDEVICE = range(7)
+(CRC_OK, CRC_EINVAL, CRC_EUNSUPPORTED, CRC_ECUDA, CRC_ETIMEOUT, CRC_ESTATE, CRC_EDEVICE,
+ CRC_ENOMEM) = range(8)
 
 
 class crc_problem(ctypes.Structure):
@@ -83,6 +85,10 @@ EXPORTS = [
      [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P, SZ, P]),
     ("crc_route_and_cache_noalloc", ctypes.c_int,
      [PP, P, P, I32, P, SZ, ctypes.POINTER(crc_trace), P]),
+    ("crc_host_staging_bytes", SZ, [PP, I32]),
+    ("crc_host_alloc", ctypes.c_int, [SZ, ctypes.POINTER(ctypes.c_void_p)]),
+    ("crc_host_free", ctypes.c_int, [P]),
+    ("crc_route_and_cache_host", ctypes.c_int, [PP, P, P, I32, I32, P, SZ, P, SZ, P, SZ, P]),
     ("crc_device_error", ctypes.c_int, []),
     ("crc_cache_scan_policy", ctypes.c_int,
      [PP, P, I32, P, SZ, ctypes.POINTER(crc_trace), I32, I32, P]),
@@ -249,6 +255,38 @@ def crc_route_and_cache(p: crc_problem, hidden_ptr: int, w_ptr: int, T: int, sta
     _ck(load().crc_route_and_cache(ctypes.byref(p), hidden_ptr, w_ptr, T, state_ptr, state_bytes,
                                    None if trace is None else ctypes.byref(trace), ws_ptr,
                                    ws_bytes, _stream(stream)), "crc_route_and_cache")
+
+
+def pinned_empty(shape, dtype):
+    """A host tensor in pinned huge-page memory from crc_host_alloc, released
+    with crc_host_free when the tensor (and every view of it) is gone."""
+    import torch
+    nbytes = math.prod(shape) * torch.empty((), dtype=dtype).element_size()
+    ptr = ctypes.c_void_p()
+    _ck(load().crc_host_alloc(max(nbytes, 1), ctypes.byref(ptr)), "crc_host_alloc")
+    addr = ptr.value
+    lib = load()
+
+    class _Pinned(ctypes.c_uint8 * max(nbytes, 1)):
+        def __del__(self):
+            lib.crc_host_free(addr)
+
+    buf = _Pinned.from_address(addr)
+    return torch.frombuffer(buf, dtype=torch.uint8)[:nbytes].view(dtype).view(shape)
+
+
+def crc_host_staging_bytes(p: crc_problem, chunk_tokens: int) -> int:
+    return int(load().crc_host_staging_bytes(ctypes.byref(p), chunk_tokens))
+
+
+def crc_route_and_cache_host(p: crc_problem, hidden_host_ptr: int, w_ptr: int, T: int,
+                             chunk_tokens: int, state_ptr: int, state_bytes: int,
+                             staging_ptr: int, staging_bytes: int, ws_ptr: int, ws_bytes: int,
+                             stream=None):
+    _ck(load().crc_route_and_cache_host(ctypes.byref(p), hidden_host_ptr, w_ptr, T, chunk_tokens,
+                                        state_ptr, state_bytes, staging_ptr, staging_bytes,
+                                        ws_ptr, ws_bytes, _stream(stream)),
+        "crc_route_and_cache_host")
 
 
 NOALLOC_SCRATCH_BYTES = 32 << 20
@@ -447,6 +485,28 @@ def route_and_cache(p: crc_problem, hidden, w_cat, state: State, trace: Trace | 
                         None if trace is None else trace.c(), workspace.data_ptr(),
                         workspace.numel() * workspace.element_size(), stream)
     return workspace
+
+
+def route_and_cache_host(p: crc_problem, hidden_host, w_cat, state: State, chunk_tokens=128,
+                         staging=None, workspace=None, stream=None):
+    """The step on hidden states [B][T][L][d] bf16 held in (pinned) host memory:
+    chunked copies overlapped with the fused step.  Returns (staging, workspace)
+    for reuse; neither may be reused before `stream` has passed this call."""
+    import torch
+    if hidden_host.device.type != "cpu" or not hidden_host.is_contiguous():
+        raise ValueError("hidden_host must be a contiguous host tensor")
+    T = hidden_host.shape[1]
+    dev = w_cat.device
+    chunk = max(1, min(chunk_tokens, T))
+    if staging is None:
+        staging = torch.empty(crc_host_staging_bytes(p, chunk), dtype=torch.uint8, device=dev)
+    if workspace is None:
+        workspace = torch.empty(crc_fused_workspace_bytes(p), dtype=torch.uint8, device=dev)
+    crc_route_and_cache_host(p, hidden_host.data_ptr(), w_cat.data_ptr(), T, chunk_tokens,
+                             state.ptr, state.nbytes, staging.data_ptr(),
+                             staging.numel() * staging.element_size(), workspace.data_ptr(),
+                             workspace.numel() * workspace.element_size(), stream)
+    return staging, workspace
 
 
 def synth_weights(L, N, d, seed=0, copy_init=False, device="cuda", stream=None):

@@ -1,8 +1,12 @@
 // C-ABI entry points of the library (declared in include/crc.h): argument
 // validation, state handling and the route-and-cache driver.
+#include <sys/mman.h>
+
 #include <atomic>
 #include <cmath>
+#include <cstdio>
 #include <cstring>
+#include <map>
 #include <mutex>
 #include <vector>
 
@@ -273,6 +277,152 @@ int crc_route_and_cache(const crc_problem* p, const uint16_t* hidden_dev,
     return CRC_OK;
 }
 
+size_t crc_host_staging_bytes(const crc_problem* p, int32_t chunk_tokens) {
+    if (check_problem(p, true) != CRC_OK || chunk_tokens < 1) return 0;
+    const size_t half = (size_t)p->B * chunk_tokens * p->L * p->d * sizeof(uint16_t);
+    return 2 * ((half + 255) / 256 * 256);
+}
+
+int crc_route_and_cache_host(const crc_problem* p, const uint16_t* hidden_host,
+                             const uint16_t* w_cat_dev, int32_t T, int32_t chunk_tokens,
+                             void* state_dev, size_t state_bytes, void* staging_dev,
+                             size_t staging_bytes, void* workspace_dev, size_t workspace_bytes,
+                             void* stream) {
+    int rc = check_problem(p, true);
+    if (rc) return rc;
+    if ((rc = check_state(p, state_dev, state_bytes))) return rc;
+    if (T < 0 || chunk_tokens < 1) return CRC_EINVAL;
+    if (T == 0) return CRC_OK;
+    if (!hidden_host || !aligned(hidden_host, 16) || !w_cat_dev || !aligned(w_cat_dev, 16))
+        return CRC_EINVAL;
+    const int chunk = chunk_tokens < T ? chunk_tokens : T;
+    if (!staging_dev || !aligned(staging_dev, 256) ||
+        staging_bytes < crc_host_staging_bytes(p, chunk))
+        return CRC_EINVAL;
+    if (!workspace_dev || !aligned(workspace_dev, 256)) return CRC_EINVAL;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t row = (size_t)p->L * p->d * sizeof(uint16_t);        // one token of one stream
+    const size_t half = crc_host_staging_bytes(p, chunk) / 2;
+    int max_pitch = 0, dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&max_pitch, cudaDevAttrMaxPitch, dev);
+    const bool two_d = (double)T * row <= (double)max_pitch;
+
+    // Copies run on a stream of the call's own, chunk i into staging half i % 2,
+    // while `stream` runs the step on chunk i - 1.  copied[j]: half j holds its
+    // chunk; done[j]: the step that read half j has finished with it.
+    cudaStream_t cs = nullptr;
+    cudaEvent_t entry = nullptr, joined = nullptr, copied[2] = {nullptr, nullptr},
+                done[2] = {nullptr, nullptr};
+    bool ok = cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) == cudaSuccess;
+    for (cudaEvent_t* e : {&entry, &joined, &copied[0], &copied[1], &done[0], &done[1]})
+        ok = ok && cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess;
+    // the staging halves may still be read by work queued earlier on `stream`
+    ok = ok && cudaEventRecord(entry, s) == cudaSuccess &&
+         cudaStreamWaitEvent(cs, entry, 0) == cudaSuccess;
+    rc = ok ? CRC_OK : CRC_ECUDA;
+    for (int t0 = 0, i = 0; rc == CRC_OK && t0 < T; t0 += chunk, ++i) {
+        const int n = (T - t0) < chunk ? (T - t0) : chunk;
+        const int j = i & 1;
+        uint8_t* buf = static_cast<uint8_t*>(staging_dev) + (size_t)j * half;
+        const uint8_t* src = reinterpret_cast<const uint8_t*>(hidden_host) + (size_t)t0 * row;
+        if (i >= 2 && cudaStreamWaitEvent(cs, done[j], 0) != cudaSuccess) rc = CRC_ECUDA;
+        // [B][n][L][d] of the chunk, stream b's tokens at pitch T * row in host memory
+        if (rc == CRC_OK && two_d) {
+            if (cudaMemcpy2DAsync(buf, (size_t)n * row, src, (size_t)T * row, (size_t)n * row,
+                                  (size_t)p->B, cudaMemcpyHostToDevice, cs) != cudaSuccess)
+                rc = CRC_ECUDA;
+        } else {
+            for (int b = 0; rc == CRC_OK && b < p->B; ++b)
+                if (cudaMemcpyAsync(buf + (size_t)b * n * row, src + (size_t)b * T * row,
+                                    (size_t)n * row, cudaMemcpyHostToDevice, cs) != cudaSuccess)
+                    rc = CRC_ECUDA;
+        }
+        if (rc == CRC_OK && (cudaEventRecord(copied[j], cs) != cudaSuccess ||
+                             cudaStreamWaitEvent(s, copied[j], 0) != cudaSuccess))
+            rc = CRC_ECUDA;
+        if (rc == CRC_OK)
+            rc = crc_route_and_cache(p, reinterpret_cast<const uint16_t*>(buf), w_cat_dev, n,
+                                     state_dev, state_bytes, nullptr, workspace_dev,
+                                     workspace_bytes, stream);
+        if (rc == CRC_OK && cudaEventRecord(done[j], s) != cudaSuccess) rc = CRC_ECUDA;
+    }
+    // everything the call queued on its copy stream is ordered before later work on `stream`
+    if (cs && joined && cudaEventRecord(joined, cs) == cudaSuccess)
+        cudaStreamWaitEvent(s, joined, 0);
+    for (cudaEvent_t e : {entry, joined, copied[0], copied[1], done[0], done[1]})
+        if (e) cudaEventDestroy(e);
+    if (cs) cudaStreamDestroy(cs);
+    return rc;
+}
+
+// Pinned host memory on transparent huge pages: anonymous mappings aligned to
+// the kernel's huge-page size, advised MADV_HUGEPAGE, faulted in one huge page
+// at a time and registered with CUDA.  The registry maps the pointer handed
+// out to its mapping.
+namespace {
+struct HostMapping {
+    void* base;
+    size_t len;
+};
+std::mutex g_host_mu;
+std::map<uintptr_t, HostMapping> g_host_maps;
+
+size_t huge_page_bytes() {
+    size_t hp = 2u << 20;
+    if (FILE* f = std::fopen("/sys/kernel/mm/transparent_hugepage/hpage_pmd_size", "r")) {
+        unsigned long long v = 0;
+        if (std::fscanf(f, "%llu", &v) == 1 && v >= 4096 && (v & (v - 1)) == 0) hp = (size_t)v;
+        std::fclose(f);
+    }
+    return hp;
+}
+}  // namespace
+
+int crc_host_alloc(size_t bytes, void** out) {
+    if (!out) return CRC_EINVAL;
+    *out = nullptr;
+    if (bytes == 0) return CRC_EINVAL;
+    const size_t hp = huge_page_bytes();
+    const size_t body = (bytes + hp - 1) / hp * hp;
+    if (body < bytes || body + hp < body) return CRC_EINVAL;
+    const size_t len = body + hp;
+    void* base = mmap(nullptr, len, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+    if (base == MAP_FAILED) return CRC_ENOMEM;
+    uint8_t* p = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(base) + hp - 1) / hp * hp);
+#ifdef MADV_HUGEPAGE
+    madvise(p, body, MADV_HUGEPAGE);    // advisory: base pages if huge pages are unavailable
+#endif
+    for (size_t o = 0; o < body; o += hp) p[o] = 0;
+    if (cudaHostRegister(p, body, cudaHostRegisterDefault) != cudaSuccess) {
+        cudaGetLastError();
+        munmap(base, len);
+        return CRC_ECUDA;
+    }
+    {
+        std::lock_guard<std::mutex> lk(g_host_mu);
+        g_host_maps[reinterpret_cast<uintptr_t>(p)] = HostMapping{base, len};
+    }
+    *out = p;
+    return CRC_OK;
+}
+
+int crc_host_free(void* ptr) {
+    if (!ptr) return CRC_OK;
+    HostMapping m;
+    {
+        std::lock_guard<std::mutex> lk(g_host_mu);
+        auto it = g_host_maps.find(reinterpret_cast<uintptr_t>(ptr));
+        if (it == g_host_maps.end()) return CRC_EINVAL;
+        m = it->second;
+        g_host_maps.erase(it);
+    }
+    const int rc = cudaHostUnregister(ptr) == cudaSuccess ? CRC_OK : CRC_ECUDA;
+    munmap(m.base, m.len);
+    return rc;
+}
+
 size_t crc_loss_workspace_bytes(const crc_problem* p, int32_t T) {
     if (check_problem(p, false) != CRC_OK || T < 1) return 0;
     const LossPlan pl = loss_plan(p->B, p->L, T);
@@ -355,6 +505,7 @@ const char* crc_strerror(int code) {
         case CRC_ETIMEOUT: return "a bounded device wait ran out";
         case CRC_ESTATE: return "state buffer too small, uninitialised or for another problem";
         case CRC_EDEVICE: return "device-side failure";
+        case CRC_ENOMEM: return "out of host memory";
         default: return "unknown error code";
     }
 }

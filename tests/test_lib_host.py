@@ -94,6 +94,40 @@ def test_router_limits_and_pointer_checks(crc):
     assert lib.crc_synth_hidden(1, 1, 1, 4, 0, 0, 1.5, 0.5, None, 16, 16, None) == crc.CRC_EINVAL
 
 
+def test_host_input_call_argument_checks(crc):
+    """crc_route_and_cache_host refuses bad arguments before it touches the GPU."""
+    lib = crc.load()
+    p = crc.problem_of(S.QWEN3_30B)
+    half = p.B * 128 * p.L * p.d * 2
+    assert crc.crc_host_staging_bytes(p, 128) == 2 * ((half + 255) // 256 * 256)
+    assert crc.crc_host_staging_bytes(p, 0) == 0
+    n = crc.crc_state_bytes(p)
+    sb = crc.crc_host_staging_bytes(p, 64)
+    ws = crc.crc_fused_workspace_bytes(p)
+    call = lambda h, T, chunk, stg, stg_bytes: lib.crc_route_and_cache_host(   # noqa: E731
+        ctypes.byref(p), h, 16, T, chunk, 256, n, stg, stg_bytes, 256, ws, None)
+    assert call(16, 0, 64, 256, sb) == crc.CRC_OK                  # T = 0: nothing queued
+    assert call(16, -1, 64, 256, sb) == crc.CRC_EINVAL
+    assert call(16, 128, 0, 256, sb) == crc.CRC_EINVAL             # chunk < 1
+    assert call(None, 128, 64, 256, sb) == crc.CRC_EINVAL          # no host buffer
+    assert call(8, 128, 64, 256, sb) == crc.CRC_EINVAL             # host buffer misaligned
+    assert call(16, 128, 64, 128, sb) == crc.CRC_EINVAL            # staging misaligned
+    assert call(16, 128, 64, 256, sb - 1) == crc.CRC_EINVAL        # staging too small
+    assert call(16, 128, 128, 256, sb) == crc.CRC_EINVAL           # ... for 128-token chunks
+    assert lib.crc_route_and_cache_host(ctypes.byref(p), 16, 16, 128, 64, 256, n - 256, 256, sb,
+                                        256, ws, None) == crc.CRC_ESTATE
+
+
+def test_host_alloc_argument_checks(crc):
+    lib = crc.load()
+    out = ctypes.c_void_p(1)
+    assert lib.crc_host_alloc(0, ctypes.byref(out)) == crc.CRC_EINVAL and not out.value
+    assert lib.crc_host_alloc(64, None) == crc.CRC_EINVAL
+    assert lib.crc_host_free(None) == crc.CRC_OK
+    assert lib.crc_host_free(4096) == crc.CRC_EINVAL         # not handed out by the library
+    assert "host memory" in crc.crc_strerror(crc.CRC_ENOMEM)
+
+
 def test_policy_scan_argument_checks(crc):
     lib = crc.load()
     p = crc.problem_of(S.QWEN3_30B)
