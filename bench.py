@@ -462,8 +462,8 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
 
     e2e = None
     if not args.no_e2e:
-        # the public call from pinned host probabilities; the means come back
-        host = torch.empty(probs.shape, dtype=torch.float32, pin_memory=True)
+        # the public call from pinned (huge-page) host probabilities; the means come back
+        host = P.pinned_empty(probs.shape, torch.float32)
         host.copy_(probs)
         out = torch.empty(2, dtype=torch.float64, pin_memory=True)
         torch.cuda.synchronize()
