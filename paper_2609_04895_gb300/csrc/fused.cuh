@@ -671,6 +671,30 @@ __global__ void __launch_bounds__(512, 1)
             }
 
             // native and Temporal heads: s^T and the Top-K set of p^R
+            // With a single accumulator, p^R is parked in the spare TMEM columns
+            // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
+            // before the Top-K selection runs.  PARK_T: the max pass also parks
+            // the raw logits (native in those columns, Temporal in shared
+            // memory) and the accumulator goes back at once; the exps are
+            // taken from the parked copies, the same values in the same order.
+            constexpr bool PARK = RC::NACC == 1 && RC::NCOL + NH <= RC::ACC_COLS;
+            const uint32_t pbase = tbase + (uint32_t)RC::NCOL;
+            auto park_t = [&](int c) {
+#pragma unroll
+                for (int q = 0; q < CW / 4; ++q)
+                    tpark[(c * CW / 4 + q) * 128 + row] =
+                        make_float4(y[4 * q], y[4 * q + 1], y[4 * q + 2], y[4 * q + 3]);
+            };
+            auto unpark_t = [&](int c) {
+#pragma unroll
+                for (int q = 0; q < CW / 4; ++q) {
+                    const float4 f = tpark[(c * CW / 4 + q) * 128 + row];
+                    y[4 * q] = f.x;
+                    y[4 * q + 1] = f.y;
+                    y[4 * q + 2] = f.z;
+                    y[4 * q + 3] = f.w;
+                }
+            };
             float mR = -INFINITY, mT = -INFINITY;
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
@@ -681,33 +705,41 @@ __global__ void __launch_bounds__(512, 1)
                 pin_cols<CW>(y);
                 mR = max_of<CW>(z, mR);
                 mT = max_of<CW>(y, mT);
+                if constexpr (Cfg::PARK_T) {
+                    tmem_put<CW>(pbase + (uint32_t)(c * CW), z);
+                    park_t(c);
+                }
+            }
+            if constexpr (Cfg::PARK_T) {
+                tmem_st_wait();
+                tc_fence_before();                        // accumulator columns fully read
+                __syncwarp();
+                if (lane == 0) release_acc(acc);
             }
             HeadExp r0, r1, t0, t1;
             r0.init(mR);
             r1.init(mR);
             t0.init(mT);
             t1.init(mT);
-            // With a single accumulator, p^R is parked in the spare TMEM columns
-            // [NCOL, NCOL + NH) so the accumulator can be handed back to the MMA
-            // before the Top-K selection runs (PAIR: already its exps, with the
-            // Temporal exps in shared memory, before s^T is formed).
-            constexpr bool PARK = RC::NACC == 1 && RC::NCOL + NH <= RC::ACC_COLS;
-            const uint32_t pbase = tbase + (uint32_t)RC::NCOL;
 #pragma unroll 1
             for (int c = 0; c < NCHK; ++c) {
-                tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
-                tmem_cols<CW>(tbase + (uint32_t)(NH + c * CW), y);
-                tmem_ld_wait();
-                pin_cols<CW>(z);
-                pin_cols<CW>(y);
+                if constexpr (Cfg::PARK_T) {
+                    tmem_cols<CW>(pbase + (uint32_t)(c * CW), z);
+                    unpark_t(c);
+                    tmem_ld_wait();
+                    pin_cols<CW>(z);
+                } else {
+                    tmem_cols<CW>(tbase + (uint32_t)(c * CW), z);
+                    tmem_cols<CW>(tbase + (uint32_t)(NH + c * CW), y);
+                    tmem_ld_wait();
+                    pin_cols<CW>(z);
+                    pin_cols<CW>(y);
+                }
                 chunk_exp(c, z, r0, r1);
                 chunk_exp(c, y, t0, t1);
                 if constexpr (Cfg::PARK_T) {
                     tmem_put<CW>(pbase + (uint32_t)(c * CW), z);
-#pragma unroll
-                    for (int q = 0; q < CW / 4; ++q)
-                        tpark[(c * CW / 4 + q) * 128 + row] =
-                            make_float4(y[4 * q], y[4 * q + 1], y[4 * q + 2], y[4 * q + 3]);
+                    park_t(c);
                 } else {
                     tmem_put<CW>(tbase + (uint32_t)(c * CW), z);
                     tmem_put<CW>(tbase + (uint32_t)(NH + c * CW), y);
@@ -718,20 +750,10 @@ __global__ void __launch_bounds__(512, 1)
             TopKAcc<KP> topk;
             topk.init();
             if constexpr (Cfg::PARK_T) {
-                tc_fence_before();                        // accumulator columns fully read
-                __syncwarp();
-                if (lane == 0) release_acc(acc);
 #pragma unroll 1
                 for (int c = 0; c < NCHK; ++c) {
                     tmem_cols<CW>(pbase + (uint32_t)(c * CW), z);
-#pragma unroll
-                    for (int q = 0; q < CW / 4; ++q) {
-                        const float4 f = tpark[(c * CW / 4 + q) * 128 + row];
-                        y[4 * q] = f.x;
-                        y[4 * q + 1] = f.y;
-                        y[4 * q + 2] = f.z;
-                        y[4 * q + 3] = f.w;
-                    }
+                    unpark_t(c);
                     tmem_ld_wait();
                     pin_cols<CW>(z);
                     retention_in_place<CW>(z, y, rR, rT);         // z = p^R, y = s^T
