@@ -255,6 +255,20 @@ int crc_route_and_cache_host(const crc_problem *p, const uint16_t *hidden_host,
                              size_t staging_bytes, void *workspace_dev, size_t workspace_bytes,
                              void *stream);
 
+/* Failure-path probe (no counterpart in the paper).  Launches one warp that
+ * waits on something that never happens -- kind 0: a flag nothing sets,
+ * through the bounded flag wait of the fused kernel; kind 1: an mbarrier
+ * phase nothing completes, through the bounded mbarrier wait of every
+ * tcgen05 kernel -- for limit_ns nanoseconds (clamped to [1 ms, 2 s], the
+ * hot-path limit being 2 s).  The expired wait latches CRC_ETIMEOUT in the
+ * state's error word, as a stalled hot-path kernel would, and the kernel
+ * returns: nothing traps or faults and the context stays usable.
+ * crc_state_read then reports CRC_ETIMEOUT.  state_dev: an initialised state
+ * of p (256-byte aligned).  Uses a two-word array compiled into the library:
+ * do not run two probes at once.  CRC_EINVAL for another kind. */
+int crc_wait_probe(const crc_problem *p, void *state_dev, size_t state_bytes, int32_t kind,
+                   uint64_t limit_ns, void *stream);
+
 /* ------------------------------------------------------------------------ */
 /* Allocation-free variant (no counterpart in the paper)                    */
 /* ------------------------------------------------------------------------ */

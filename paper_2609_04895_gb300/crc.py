@@ -88,6 +88,7 @@ EXPORTS = [
     ("crc_host_staging_bytes", SZ, [PP, I32]),
     ("crc_host_alloc", ctypes.c_int, [SZ, ctypes.POINTER(ctypes.c_void_p)]),
     ("crc_host_free", ctypes.c_int, [P]),
+    ("crc_wait_probe", ctypes.c_int, [PP, P, SZ, I32, U64, P]),
     ("crc_route_and_cache_host", ctypes.c_int, [PP, P, P, I32, I32, P, SZ, P, SZ, P, SZ, P]),
     ("crc_device_error", ctypes.c_int, []),
     ("crc_cache_scan_policy", ctypes.c_int,

@@ -65,7 +65,7 @@ __device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
 
 // Single-thread bounded wait for *p >= target.  False on timeout or abort.
 __device__ __forceinline__ bool wait_geq(const uint32_t* p, uint32_t target, uint32_t* abort_flag,
-                                         uint32_t* err) {
+                                         uint32_t* err, uint64_t limit_ns = kWaitLimitNs) {
     if (ld_acquire_u32(p) >= target) return true;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
@@ -75,7 +75,7 @@ __device__ __forceinline__ bool wait_geq(const uint32_t* p, uint32_t target, uin
             if (ld_acquire_u32(p) >= target) return true;
         }
         if (ld_acquire_u32(abort_flag)) return false;
-        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+        if (globaltimer_ns() - t0 > limit_ns) {
             latch_error(err, CRC_ETIMEOUT);
             atomicExch(abort_flag, 1u);
             return false;

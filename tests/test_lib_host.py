@@ -128,6 +128,16 @@ def test_host_alloc_argument_checks(crc):
     assert "host memory" in crc.crc_strerror(crc.CRC_ENOMEM)
 
 
+def test_wait_probe_argument_checks(crc):
+    lib = crc.load()
+    p = crc.problem_of(S.TINY)
+    n = crc.crc_state_bytes(p)
+    assert lib.crc_wait_probe(ctypes.byref(p), None, n, 0, 10**7, None) == crc.CRC_EINVAL
+    assert lib.crc_wait_probe(ctypes.byref(p), 128, n, 0, 10**7, None) == crc.CRC_EINVAL
+    assert lib.crc_wait_probe(ctypes.byref(p), 256, n, 2, 10**7, None) == crc.CRC_EINVAL
+    assert lib.crc_wait_probe(ctypes.byref(p), 256, n - 1, 0, 10**7, None) == crc.CRC_EINVAL
+
+
 def test_policy_scan_argument_checks(crc):
     lib = crc.load()
     p = crc.problem_of(S.QWEN3_30B)
