@@ -1,8 +1,9 @@
-"""Failure detection on the GPU without a fault: a bounded wait that runs out
-(a flag nothing sets; an mbarrier phase nothing completes) latches
-CRC_ETIMEOUT in the state, the host reads it through crc_state_read, the
-kernel has returned within about the wait limit, and the context still runs
-the hot path correctly afterwards."""
+"""Failure detection on the GPU without a fault, and checkpoint / resume of
+the state.  A bounded wait that runs out (a flag nothing sets; an mbarrier
+phase nothing completes) latches CRC_ETIMEOUT in the state, the host reads it
+through crc_state_read, the kernel has returned within about the wait limit,
+and the context still runs the hot path correctly afterwards.  A state copied
+to the host and restored elsewhere continues the streams exactly."""
 import ctypes
 import time
 
@@ -53,3 +54,33 @@ def test_expired_wait_reports_timeout_and_context_survives(C, kind):
     r2 = s2.read(want_caches=True)
     assert r1["error"] == 0 and r1["tokens"] == w.T
     assert (r1["cache_bits"] == r2["cache_bits"]).all() and r1["misses"] == r2["misses"]
+
+
+def test_checkpoint_to_host_and_resume_elsewhere(C):
+    """Checkpoint / resume: the state is position-independent bytes.  Copy it
+    to the host after T1 tokens, restore it into a fresh buffer (another
+    address), continue with the remaining tokens: the same final caches,
+    counters and carried scores as one uninterrupted call."""
+    w = S.QWEN3_30B.with_(B=2, T=300, L=3, d=128)
+    p = C.problem_of(w)
+    Wd = C.synth_weights(w.L, w.N, w.d, seed=7)
+    hd, _ = C.synth_hidden(w.B, w.T, w.L, w.d, seed=8)
+    ws = torch.empty(C.crc_fused_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    whole = C.State(p)
+    C.route_and_cache(p, hd, Wd, whole, workspace=ws)
+    ref = whole.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    T1 = 170
+    first = C.State(p)
+    C.route_and_cache(p, hd[:, :T1].contiguous(), Wd, first, workspace=ws)
+    saved = first.buf.cpu()                                # checkpoint
+    del first
+    resumed = C.State(p)
+    resumed.buf.copy_(saved)                               # resume into a new buffer
+    assert resumed.ptr != saved.data_ptr()
+    C.route_and_cache(p, hd[:, T1:].contiguous(), Wd, resumed, workspace=ws)
+    got = resumed.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    for k, v in ref.items():
+        if hasattr(v, "shape"):
+            assert (v == got[k]).all(), k
+        else:
+            assert v == got[k], k
