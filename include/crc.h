@@ -201,7 +201,11 @@ size_t crc_fused_workspace_bytes(const crc_problem *p);
  * the call is one fused kernel; for N = 128 with 128-token tiles of one stream
  * (T > 64) and an even stream count its GEMM runs on CTA pairs (clusters of
  * two, tcgen05 cta_group::2), otherwise one CTA per tile, with the same
- * results.  Without that workspace, workspace_dev holds the scores of one
+ * results.  The pair kernel is a cooperative cluster launch; with the
+ * environment variable CRC_PLAIN_CLUSTER_LAUNCH=1 (read once per process) it
+ * is launched without the cooperative attribute, for kernel profilers that
+ * cannot replay cooperative cluster launches (same kernel, same grid, which
+ * fits the GPU at once; a stall would end in CRC_ETIMEOUT).  Without that workspace, workspace_dev holds the scores of one
  * chunk of tokens, the chunk length being the largest that fits (at least one
  * token must fit, see crc_workspace_bytes).  256-byte alignment for the
  * workspace. */

@@ -4,11 +4,20 @@
 #pragma once
 
 #include <algorithm>
+#include <cstdlib>
 
 #include "crc_internal.h"
 #include "fused.cuh"
 
 namespace crc {
+
+inline bool plain_cluster_launch() {
+    static const bool on = [] {
+        const char* v = std::getenv("CRC_PLAIN_CLUSTER_LAUNCH");
+        return v && v[0] == '1' && v[1] == '\0';
+    }();
+    return on;
+}
 
 struct FusedPlan {
     int SB, TB, n_bg, n_tb, tiles_per_tb, num_tiles, ring, n_items;
@@ -140,7 +149,12 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
         c.dynamicSmemBytes = Cfg::SMEM_BYTES;
         c.stream = stream;
         c.attrs = at;
-        c.numAttrs = 2;
+        // CRC_PLAIN_CLUSTER_LAUNCH=1 drops the cooperative attribute so that a
+        // kernel profiler, which cannot replay a cooperative cluster launch,
+        // can run the same kernel; the grid still fits the GPU at once (the
+        // occupancy query above), and were it ever not co-resident, the bounded
+        // waits would end the call with CRC_ETIMEOUT
+        c.numAttrs = plain_cluster_launch() ? 1 : 2;
         {
             ProfScope prof(CRC_KERNEL_FUSED, stream);
             e = cudaLaunchKernelExC(&c, (const void*)kern, args);
