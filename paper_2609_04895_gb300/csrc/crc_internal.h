@@ -62,7 +62,7 @@ int launch_policy_scan(const crc_problem& p, const float* scores, int T, void* s
 int launch_fused_n128(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                       void* state, void* workspace, cudaStream_t stream);
 
-// Soft Top-B coverage losses (loss.cu): the task split over token chunks and
+// Soft Top-B coverage losses (loss.cu): the work split over token chunks and
 // the launch; workspace = per-task sums, 16 bytes per task.
 struct LossPlan {
     int nchunks, chunk;
