@@ -463,7 +463,7 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
     e2e = None
     if not args.no_e2e:
         # the public call from pinned (huge-page) host probabilities; the means come back
-        host = P.pinned_empty(probs.shape, torch.float32)
+        host, host_mem = pinned_host(P, probs.shape, torch.float32)
         host.copy_(probs)
         out = torch.empty(2, dtype=torch.float64, pin_memory=True)
         torch.cuda.synchronize()
@@ -480,7 +480,7 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
         ems = max_over_ranks(f0.elapsed_time(f1), world, dev)
         e2e = {"value": job_rate(w.units, world, ems / args.steps), "unit": LOSS_UNIT,
                "h2d_bytes_per_step": int(probs.numel() * 4), "d2h_bytes_per_step": 16,
-               "ms_per_step": ems / args.steps}
+               "ms_per_step": ems / args.steps, "host_memory": host_mem}
         del host
 
     cpu = None
@@ -935,7 +935,7 @@ def end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all
     import torch
     import torch.distributed as dist
     hd = held.pop()
-    h_host = P.pinned_empty(hd.shape, hd.dtype)
+    h_host, host_mem = pinned_host(P, hd.shape, hd.dtype)
     h_host.copy_(hd)
     del hd
     torch.cuda.empty_cache()
@@ -964,9 +964,19 @@ def end_to_end(args, P, C, w, p, held, Wd, st, ws, stream, dev, world, units_all
             "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": int(256 + p.B * p.L * 64),
             "ms_per_step": 1000 * dt / args.steps,
-            "call": f"crc_route_and_cache_host, {chunk}-token chunks",
+            "call": f"crc_route_and_cache_host, {chunk}-token chunks", "host_memory": host_mem,
             "host_link_gbs": host_link_gbs(h_host, staging, stream),
             "h2d_gbs": h2d / (dt / args.steps) / 1e9}
+
+
+def pinned_host(P, shape, dtype):
+    """Pinned host memory for an end-to-end input: crc_host_alloc's huge pages,
+    else (registration refused on this host) cudaHostAlloc's, named in the line."""
+    import torch
+    try:
+        return P.pinned_empty(shape, dtype), "crc_host_alloc (huge pages)"
+    except P.CrcError as e:
+        return torch.empty(shape, dtype=dtype, pin_memory=True), f"cudaHostAlloc ({e})"
 
 
 def host_link_gbs(h_host, dev_buf, stream) -> float:
