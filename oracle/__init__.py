@@ -281,7 +281,7 @@ def bits_to_sets(cache_bits: np.ndarray, N: int):
 
 
 def refine(in_cache: np.ndarray, sST, C: int, R: int, dtype=np.float64):
-    """Algorithm 2 lines 3-13 on a copy of in_cache.  Returns (new_in_cache, proactive, margin)."""
+    """Algorithm 2's refinement loop on a copy of in_cache.  Returns (new_in_cache, proactive, margin)."""
     dt = np.dtype(dtype)
     sfx = "f64" if dt == np.float64 else "f32"
     ic = np.array(in_cache, dtype=np.uint8)

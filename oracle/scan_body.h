@@ -49,7 +49,7 @@ static int FN(argmin_last)(const REAL *s, const uint8_t *member, int N, double *
 }
 
 /*
- * Algorithm 2, lines 3-13: pre-access refinement of a cache with priorities
+ * Algorithm 2, the refinement loop: pre-access refinement of a cache with priorities
  * sST (s^ST_{t,l}).  A = Top_R(sST) over all N experts; each candidate, in
  * descending order, is skipped when resident, inserted when the cache has a
  * free slot, else replaces the lowest resident only when strictly higher.
@@ -145,7 +145,7 @@ int FN(oracle_step)(int N, int K, int C, int R, int t,
     double margin = INFINITY, g;
     int proactive = 0;
 
-    /* lines 1-13: pre-access refinement (full mode, t >= 1) */
+    /* Algorithm 2, refinement: pre-access refinement (full mode, t >= 1) */
     if (R > 0 && t >= 1) {
         for (int e = 0; e < N; e++) {
             REAL a = aT[e];                 /* a^T = p^R_{t-1,l} + p^T_{t-1,l} */
@@ -154,7 +154,7 @@ int FN(oracle_step)(int N, int K, int C, int R, int t,
         proactive = FN(oracle_refine)(N, C, R, sST, in_cache, count, &margin);
     }
 
-    /* line 14: native Top-K on p^R (the set boundary K/K+1 is the decision;
+    /* Algorithm 2, access: native Top-K on p^R (the set boundary K/K+1 is the decision;
      * the order inside the set only orders the trace) */
     FN(order_desc)(pR, N, ord);
     uint8_t inS[ORACLE_MAX_N];
@@ -168,10 +168,10 @@ int FN(oracle_step)(int N, int K, int C, int R, int t,
         if (g < margin) margin = g;
     }
 
-    /* line 16: s^T = p^R + p^T */
+    /* Algorithm 2, retention score: s^T = p^R + p^T */
     for (int e = 0; e < N; e++) sT[e] = pR[e] + pT[e];
 
-    /* lines 15 and 17: demand-load S \ C~, then UpdateCache (Algorithm 1) */
+    /* Algorithm 2, demand load of S \ C~, then UpdateCache (Algorithm 1) */
     int misses = FN(oracle_update_cache)(N, C, sT, inS, in_cache, count, &margin);
     for (int e = 0; e < N; e++) aT[e] = sT[e];
 
