@@ -219,6 +219,56 @@ def hidden_stream(seed: int, b: int, T: int, L: int, d: int, rho_t: float, rho_l
     return out
 
 
+class HiddenWalk:
+    """One stream's hidden states drawn unit by unit in causal order
+    (t = 0, 1, ...; l = 0 .. L-1 within a token), with the definition of
+    ``hidden_stream``: ``draw(t, l, attempt)`` proposes h[t, l] from the
+    innovation of that attempt without changing the walk, ``accept`` keeps
+    the proposal.  A test that redraws a unit's innovation (to move a draw
+    away from an unwanted event) walks the same field ``hidden_stream``
+    produces when given the accepted attempts as its re-draw table."""
+
+    def __init__(self, seed: int, b: int, L: int, d: int, rho_t: float, rho_l: float):
+        if d % 2:
+            raise ValueError("d must be even")
+        self.seed, self.b, self.L, self.d = seed, b, L, d
+        self.rt, self.st = ar_constants(rho_t)
+        self.rl, self.sl = ar_constants(rho_l)
+        self.h_prev = None            # h[t-1, :] fp32 [L][d]
+        self.h_cur = np.empty((L, d), np.float32)
+        self.g_prev = None            # g[t, l-1] fp32 [d]
+        self._t = -1
+        self._eps0 = None             # innovations of attempt 0 for token t, [L][d]
+
+    def _eps(self, t: int, l: int, attempt: int) -> np.ndarray:
+        if attempt == 0:
+            if self._t != t:
+                self._eps0 = _innovations(self.seed, self.b, [t], self.L, self.d)[0]
+                self._t = t
+            return self._eps0[l]
+        j = np.arange(self.d // 2, dtype=np.uint32)
+        c3 = np.uint32(self.b) | (np.uint32(attempt) << np.uint32(16))
+        ev, od = normal_pairs(j, np.uint32(l), np.uint32(t), c3, self.seed, TAG_HIDDEN)
+        e = np.empty(self.d, np.float32)
+        e[0::2] = ev
+        e[1::2] = od
+        return e
+
+    def draw(self, t: int, l: int, attempt: int = 0):
+        """Proposal for unit (t, l): (bf16 bits [d], state to pass to accept)."""
+        eps = self._eps(t, l, attempt)
+        g = eps.copy() if l == 0 else (self.rl * self.g_prev) + (self.sl * eps)
+        h = g.copy() if self.h_prev is None else (self.rt * self.h_prev[l]) + (self.st * g)
+        return bf16_rne_bits(h), (t, l, g, h)
+
+    def accept(self, state) -> None:
+        t, l, g, h = state
+        self.g_prev = g
+        self.h_cur[l] = h
+        if l == self.L - 1:
+            self.h_prev = self.h_cur.copy()
+
+
 def hidden(w: Workload, seed: int = 0, streams=None, T: int | None = None,
            attempts: np.ndarray | None = None) -> np.ndarray:
     """bf16 bits [len(streams)][T][L][d] (all streams by default)."""

@@ -74,15 +74,21 @@ typedef struct crc_problem {
 
 /* Optional per-access trace of one call, device pointers, each may be NULL.
  * T is the call's token count and t the token index within the call.  The
- * cache sets are bitmasks of NW = ceil(N / 32) words per access (expert e is
- * bit e % 32 of word e / 32); they are written by the method's scan only
- * (crc_cache_scan, crc_route_and_cache), not by the comparison policies. */
+ * sets are bitmasks of NW = ceil(N / 32) words per access (expert e is bit
+ * e % 32 of word e / 32); the cache sets and the Top-K set are written by the
+ * method's scan only (crc_cache_scan, crc_route_and_cache), not by the
+ * comparison policies.  The native Top-K comes in two forms: topk_dev in rank
+ * order (p^R descending, ties to the lower index), and topk_set_dev, the same
+ * experts as a set, which is all that the cache decisions use (Sec. 2:
+ * S = TopK(p^R) is a set).  crc_route_and_cache runs as one fused kernel
+ * with any trace that does not ask for topk_dev (see there). */
 typedef struct crc_trace {
     uint8_t *topk_dev;       /* [B][T][L][K] native Top-K, rank order          */
     uint8_t *misses_dev;     /* [B][T][L] demand misses |S \ C~|               */
     uint8_t *proactive_dev;  /* [B][T][L] proactive loads of the refinement    */
     uint32_t *cache_mid_dev; /* [B][T][L][NW] cache after Algorithm 2 (C~)     */
     uint32_t *cache_after_dev; /* [B][T][L][NW] cache after UpdateCache      */
+    uint32_t *topk_set_dev;  /* [B][T][L][NW] native Top-K S as a set          */
 } crc_trace;
 
 /* Totals over all streams and layers since crc_state_init (Sec. 4.1). */
@@ -187,18 +193,18 @@ size_t crc_workspace_bytes(const crc_problem *p, int32_t chunk_tokens);
 
 /* Workspace bytes with which crc_route_and_cache runs as ONE fused kernel
  * (router heads on the tensor cores and the scan together; the router scores
- * then only pass through an L2-sized ring of tiles in the workspace).  The
- * fused kernel serves calls without a trace and with K <= 8 and 16 <= N <= 128;
- * other calls, or smaller workspaces, take the chunked two-kernel path.
- * 0 if p is invalid. */
+ * then only pass through a ring of tiles in the workspace).  The fused kernel
+ * serves calls with K <= 8 and 16 <= N <= 128 whose trace, if any, does not
+ * ask for the Top-K in rank order (crc_trace.topk_dev); other calls, or
+ * smaller workspaces, take the chunked two-kernel path.  0 if p is invalid. */
 size_t crc_fused_workspace_bytes(const crc_problem *p);
 
 /* The whole step: router heads and cache simulation over T tokens, the
  * same results as crc_route_scores followed by crc_cache_scan (bit for bit).
  * hidden_dev bf16 [B][T][L][d]; w_cat_dev bf16 [L][3N][d] (the S head is
  * not computed when R = 0).  The router scores never leave the workspace.
- * With workspace_bytes >= crc_fused_workspace_bytes(p) (and no trace, K <= 8)
- * the call is one fused kernel; for N = 128 with 128-token tiles of one stream
+ * With workspace_bytes >= crc_fused_workspace_bytes(p), K <= 8 and a trace
+ * that leaves topk_dev NULL (or no trace) the call is one fused kernel; for N = 128 with 128-token tiles of one stream
  * (T > 64) and an even stream count its GEMM runs on CTA pairs (clusters of
  * two, tcgen05 cta_group::2), otherwise one CTA per tile, with the same
  * results.  The pair kernel is a cooperative cluster launch; with the

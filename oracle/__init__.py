@@ -62,7 +62,7 @@ def lib():
                 f.argtypes = [i, i, i, i, i, P, P, P, P, P, P, P, P, P, P]
                 f.restype = i
                 f = getattr(L, f"oracle_scan_{sfx}")
-                f.argtypes = [i, i, i, i, i, i, i, P, P, P, P, P, P, P, P, i]
+                f.argtypes = [i, i, i, i, i, i, i, P, P, P, P, P, P, P, P, i, i]
                 f.restype = i
                 f = getattr(L, f"oracle_refine_{sfx}")
                 f.argtypes = [i, i, i, P, P, P, P]
@@ -113,12 +113,17 @@ def router_probs(hidden_bits: np.ndarray, w_bits: np.ndarray, N: int, H: int = 3
 
 
 def scan(probs: np.ndarray, K: int, C: int, R: int, trace: bool = True,
-         margins: bool = False, nthreads: int | None = None) -> dict:
+         margins: bool = False, nthreads: int | None = None,
+         exact_ties_exempt: bool = False) -> dict:
     """Literal Algorithm 2 + 1 over [B][T][L][3][N] probabilities.
 
     fp64 input runs the fp64 scan; fp32 input runs the fp32 scan (every sum
     and comparison in fp32).  Returns the trace, the final caches and the
     per-(stream, layer) counters (hits, demand misses, proactive loads).
+    margins: each access's decision margin, the smallest relative gap between
+    the two scores of any decision it took; exact_ties_exempt leaves gaps of
+    exactly zero out of it (ties built on purpose, broken by index on every
+    side).
     """
     if probs.dtype == np.float64:
         sfx = "f64"
@@ -142,7 +147,8 @@ def scan(probs: np.ndarray, K: int, C: int, R: int, trace: bool = True,
     rc = getattr(lib(), f"oracle_scan_{sfx}")(
         B, T, L, N, K, C, R, _ptr(p), _ptr(res["topk"]), _ptr(res["misses"]),
         _ptr(res["proactive"]), _ptr(res["margins"]), _ptr(res["cache_bits"]),
-        _ptr(res["aT"]), _ptr(res["counters"]), nthreads or default_threads())
+        _ptr(res["aT"]), _ptr(res["counters"]), nthreads or default_threads(),
+        int(exact_ties_exempt))
     if rc != 0:
         raise ValueError("oracle_scan rejected the sizes")
     return res
@@ -262,11 +268,13 @@ def load_time(D: float, P: float, T: float, c_exp: float, eta: float) -> float:
 
 
 def run(hidden_bits: np.ndarray, w_bits: np.ndarray, N: int, K: int, C: int, R: int,
-        margins: bool = True, nthreads: int | None = None) -> dict:
+        margins: bool = True, nthreads: int | None = None,
+        exact_ties_exempt: bool = False) -> dict:
     """End-to-end fp64 oracle: router probabilities then the scan."""
     H = 3 if R > 0 else 2
     p = router_probs(hidden_bits, w_bits, N, H, nthreads)
-    res = scan(p, K, C, R, trace=True, margins=margins, nthreads=nthreads)
+    res = scan(p, K, C, R, trace=True, margins=margins, nthreads=nthreads,
+               exact_ties_exempt=exact_ties_exempt)
     res["probs"] = p
     return res
 

@@ -146,9 +146,17 @@ void oracle_router_probs(int B, int T, int L, int N, int d, int H,
 /* ------------------------------------------------------------------------ */
 /* cache scan, one body for two precisions                                   */
 /* ------------------------------------------------------------------------ */
+/* Decision margins: the relative gap |a - b| / max(|a|, |b|) between the two
+ * scores a decision compares.  A test that builds exact ties on purpose (two
+ * experts with identical weight rows have identical scores on every side,
+ * and every side breaks such a tie by the same index rule) may exempt gaps of
+ * exactly zero; the setting is per thread, made by the scan for its workers. */
+static _Thread_local int exact_ties_exempt;
+
 static double rel_gap(double a, double b)
 {
     double m = fabs(a) > fabs(b) ? fabs(a) : fabs(b);
+    if (a == b && exact_ties_exempt) return INFINITY;
     if (m == 0.0) return 0.0;
     return fabs(a - b) / m;
 }

@@ -191,6 +191,7 @@ typedef struct {
     uint64_t *counters;
     int b_begin, b_end;
     int status;
+    int ties_exempt;
 } FN(scan_job);
 
 static void *FN(scan_worker)(void *arg)
@@ -203,6 +204,7 @@ static void *FN(scan_worker)(void *arg)
     REAL *aT = (REAL *)calloc((size_t)L * N, sizeof(REAL));
     int topk[ORACLE_MAX_N];
     j->status = 0;
+    exact_ties_exempt = j->ties_exempt;
     for (int b = j->b_begin; b < j->b_end; b++) {
         memset(in_cache, 0, (size_t)L * N);
         memset(count, 0, sizeof(int) * (size_t)L);
@@ -249,6 +251,7 @@ static void *FN(scan_worker)(void *arg)
         }
     }
 done:
+    exact_ties_exempt = 0;
     free(in_cache);
     free(count);
     free(aT);
@@ -261,12 +264,13 @@ done:
  * Outputs (any trace pointer may be NULL): topk [B][T][L][K] in rank order,
  * misses / proactive [B][T][L], margins [B][T][L], cache_bits [B][L][ceil(N/32)],
  * aT_out [B][L][N] (s^T of the last token), counters [B][L][3] = hits,
- * demand misses, proactive loads.  Returns 0 or -1.
+ * demand misses, proactive loads.  ties_exempt: gaps of exactly zero do not
+ * lower the margins (ties built on purpose).  Returns 0 or -1.
  */
 int FN(oracle_scan)(int B, int T, int L, int N, int K, int C, int R,
                     const REAL *probs, uint8_t *topk, uint8_t *misses,
                     uint8_t *proactive, double *margins, uint32_t *cache_bits,
-                    REAL *aT_out, uint64_t *counters, int nthreads)
+                    REAL *aT_out, uint64_t *counters, int nthreads, int ties_exempt)
 {
     if (B < 0 || T < 0 || L < 1 || N < 1 || N > ORACLE_MAX_N || K < 1 || K > N ||
         C < K || C > N || R < 0)
@@ -280,7 +284,7 @@ int FN(oracle_scan)(int B, int T, int L, int N, int K, int C, int R,
     for (int k = 0; k < nthreads; k++) {
         FN(scan_job) jj = {B, T, L, N, K, C, R, probs, topk, misses, proactive,
                            margins, cache_bits, aT_out, counters,
-                           k * per, (k + 1) * per < B ? (k + 1) * per : B, 0};
+                           k * per, (k + 1) * per < B ? (k + 1) * per : B, 0, ties_exempt};
         jobs[k] = jj;
     }
     if (nthreads == 1) {

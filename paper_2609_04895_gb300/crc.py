@@ -32,7 +32,7 @@ class crc_problem(ctypes.Structure):
 class crc_trace(ctypes.Structure):
     _fields_ = [("topk_dev", ctypes.c_void_p), ("misses_dev", ctypes.c_void_p),
                 ("proactive_dev", ctypes.c_void_p), ("cache_mid_dev", ctypes.c_void_p),
-                ("cache_after_dev", ctypes.c_void_p)]
+                ("cache_after_dev", ctypes.c_void_p), ("topk_set_dev", ctypes.c_void_p)]
 
 
 class crc_transfer(ctypes.Structure):
@@ -380,22 +380,30 @@ class Trace:
     proactive: object
     cache_mid: object = None
     cache_after: object = None
+    topk_set: object = None
 
     @staticmethod
-    def alloc(p: crc_problem, T: int, device="cuda", caches: bool = False) -> "Trace":
+    def alloc(p: crc_problem, T: int, device="cuda", caches: bool = False,
+              rank_order: bool = True, topk_set: bool = False) -> "Trace":
         """caches: also the cache sets after the refinement and after the update
-        ([B][T][L][NW] uint32 bitmasks)."""
+        ([B][T][L][NW] uint32 bitmasks); rank_order=False leaves out the Top-K
+        in rank order (such a trace keeps crc_route_and_cache on its fused
+        kernel); topk_set: the Top-K as a [B][T][L][NW] bitmask."""
         import torch
         nw = (p.N + 31) // 32
-        mk = (lambda: torch.zeros((p.B, T, p.L, nw), dtype=torch.int32, device=device)) \
-            if caches else (lambda: None)
-        return Trace(torch.zeros((p.B, T, p.L, p.K), dtype=torch.uint8, device=device),
+
+        def words(on):
+            return torch.zeros((p.B, T, p.L, nw), dtype=torch.int32, device=device) if on else None
+
+        return Trace(torch.zeros((p.B, T, p.L, p.K), dtype=torch.uint8, device=device)
+                     if rank_order else None,
                      torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device),
-                     torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device), mk(), mk())
+                     torch.zeros((p.B, T, p.L), dtype=torch.uint8, device=device),
+                     words(caches), words(caches), words(topk_set))
 
     def c(self) -> crc_trace:
         return crc_trace(_ptr(self.topk), _ptr(self.misses), _ptr(self.proactive),
-                         _ptr(self.cache_mid), _ptr(self.cache_after))
+                         _ptr(self.cache_mid), _ptr(self.cache_after), _ptr(self.topk_set))
 
 
 def transfer_plan(p: crc_problem, cache_mid, cache_after, slot_expert=None, start=None):

@@ -44,7 +44,8 @@ int check_state(const crc_problem* p, const void* state, size_t bytes) {
 int check_trace(const crc_trace* tr) {
     // every trace pointer may be null; bytes need no alignment, mask words 4 bytes
     if (tr && ((tr->cache_mid_dev && !aligned(tr->cache_mid_dev, 4)) ||
-               (tr->cache_after_dev && !aligned(tr->cache_after_dev, 4))))
+               (tr->cache_after_dev && !aligned(tr->cache_after_dev, 4)) ||
+               (tr->topk_set_dev && !aligned(tr->topk_set_dev, 4))))
         return CRC_EINVAL;
     return CRC_OK;
 }
@@ -254,11 +255,13 @@ int crc_route_and_cache(const crc_problem* p, const uint16_t* hidden_dev,
     if (!hidden_dev || !w_cat_dev || !aligned(hidden_dev, 16) || !aligned(w_cat_dev, 16))
         return CRC_EINVAL;
     if (!workspace_dev || !aligned(workspace_dev, 256)) return CRC_EINVAL;
+    if ((rc = check_trace(trace))) return rc;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const bool traced = trace && (trace->topk_dev || trace->misses_dev || trace->proactive_dev ||
-                                  trace->cache_mid_dev || trace->cache_after_dev);
-    if (!traced) {
-        rc = launch_fused(*p, hidden_dev, w_cat_dev, T, state_dev, workspace_dev, workspace_bytes, s);
+    // the fused kernel knows the Top-K as a set only: a trace in rank order
+    // takes the two-kernel path
+    if (!(trace && trace->topk_dev)) {
+        rc = launch_fused(*p, hidden_dev, w_cat_dev, T, state_dev, workspace_dev, workspace_bytes,
+                          trace, s);
         if (rc != CRC_EUNSUPPORTED) return rc;
     }
     const size_t per_token = crc_workspace_bytes(p, 1);

@@ -32,6 +32,7 @@ struct ScanArgs {
     uint8_t* trace_pro;      // [B][T][L] or null
     uint32_t* trace_mid;     // [B][T][L][NW] cache after the refinement, or null
     uint32_t* trace_after;   // [B][T][L][NW] cache after UpdateCache, or null
+    uint32_t* trace_sel;     // [B][T][L][NW] native Top-K set, or null
     int trace_T, trace_t0;   // trace arrays span trace_T tokens; this call starts at trace_t0
     int B, T, L, N, K, C, R;
 };
@@ -417,7 +418,8 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
                                           int R, bool have_sel, uint32_t sel_in,
                                           uint8_t* topk_out, uint8_t* miss_out,
                                           uint8_t* pro_out, uint32_t* mid_out = nullptr,
-                                          uint32_t* after_out = nullptr, int N = 0) {
+                                          uint32_t* after_out = nullptr, int N = 0,
+                                          uint32_t* sel_out = nullptr) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
     float sT[V];
 #pragma unroll
@@ -456,6 +458,7 @@ __device__ __forceinline__ void scan_step(ChainRegs<V>& cr, const float (&pR)[V]
         pro = scan_apply<V, ALL_VALID>(cr, sT, pS, refine, valid, lane, K, C, R, sel, &nD);
     }
     if (after_out) store_cache_words<V>(cr.cache, lane, N, after_out);
+    if (sel_out) store_cache_words<V>(sel, lane, N, sel_out);
     if (want_topk && lane < K) topk_out[lane] = (uint8_t)my_topk;
     if (lane == 0) {
         if (miss_out) *miss_out = (uint8_t)nD;
@@ -560,7 +563,7 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
                          a.trace_pro ? a.trace_pro + unit : nullptr,
                          a.trace_mid ? a.trace_mid + unit * (size_t)((N + 31) >> 5) : nullptr,
                          a.trace_after ? a.trace_after + unit * (size_t)((N + 31) >> 5) : nullptr,
-                         N);
+                         N, a.trace_sel ? a.trace_sel + unit * (size_t)((N + 31) >> 5) : nullptr);
             cR = nR;
             cT = nT;
             cS = nS;

@@ -48,19 +48,24 @@ bool make_weight_map(CUtensorMap* m, const uint16_t* w, int L, int N3, int d, in
 // problem, and the launch (CRC_EUNSUPPORTED when the problem is outside it).
 size_t fused_workspace_bytes(const crc_problem& p);
 int launch_fused(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                 void* state, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+                 void* state, void* workspace, size_t workspace_bytes, const crc_trace* trace,
+                 cudaStream_t stream);
 int launch_fused_n16(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                     void* state, void* workspace, cudaStream_t stream);
+                     void* state, void* workspace, const crc_trace* trace,
+                     cudaStream_t stream);
 int launch_fused_n32(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                     void* state, void* workspace, cudaStream_t stream);
+                     void* state, void* workspace, const crc_trace* trace,
+                     cudaStream_t stream);
 int launch_fused_n64(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                     void* state, void* workspace, cudaStream_t stream);
+                     void* state, void* workspace, const crc_trace* trace,
+                     cudaStream_t stream);
 // Cache scan under a comparison policy (policy_scan.cuh).
 int launch_policy_scan(const crc_problem& p, const float* scores, int T, void* state,
                        const crc_trace* trace, int trace_T, int trace_t0, int policy,
                        int lambda2, cudaStream_t stream);
 int launch_fused_n128(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                      void* state, void* workspace, cudaStream_t stream);
+                      void* state, void* workspace, const crc_trace* trace,
+                     cudaStream_t stream);
 
 // Soft Top-B coverage losses (loss.cu): the work split over token chunks and
 // the launch; workspace = per-task sums, 16 bytes per task.

@@ -43,6 +43,13 @@ struct FusedArgs {
     uint32_t* prog;         // [B*L] token blocks finished per chain
     uint8_t* ring_base;
     size_t slot_bytes;
+    // optional per-access trace of the call ([B][T][L] bytes, [B][T][L][NW]
+    // bitmasks), each null when not wanted
+    uint8_t* tr_miss;
+    uint8_t* tr_pro;
+    uint32_t* tr_mid;
+    uint32_t* tr_after;
+    uint32_t* tr_sel;
 };
 
 // Ring slot layout for tile rows r in [0,128): Top-K mask words [NW][128] u32,
@@ -184,6 +191,8 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
     const bool has = valid != 0u;
     const bool want_s = a.R > 0;
     const uint32_t e0 = (uint32_t)lane * V;
+    const int NW = (N + 31) >> 5;
+    const bool traced = a.tr_miss || a.tr_pro || a.tr_mid || a.tr_after || a.tr_sel;
     while (true) {
         uint32_t item = 0u;
         if (lane == 0) item = atomicAdd(&a.ctl[0], 1u);
@@ -285,9 +294,27 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
             if (tbi + 1 < steps) fetch(tbi + 1, nT, nS, nsel);
             if ((tbi & 7) == 0) prefetch_rows(tbi + 24);
             const bool refine = want_s && tbi >= refine_from;
+            const uint32_t sel = (csel >> (e0 & 31)) & ((1u << V) - 1u);
             int nD;
-            scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R,
-                                     (csel >> (e0 & 31)) & ((1u << V) - 1u), &nD);
+            if (traced) {
+                // the refinement on its own, so the cache between the phases is seen
+                const size_t unit = ((size_t)b * a.T + tb * a.TB + tbi) * L + l;
+                const int pro = refine ? scan_refine<V, ALL_VALID>(cr, cS, valid, lane, a.C, a.R)
+                                       : 0;
+                if (a.tr_mid) store_cache_words<V>(cr.cache, lane, N, a.tr_mid + unit * NW);
+                scan_apply<V, ALL_VALID>(cr, cT, cS, false, valid, lane, a.K, a.C, a.R, sel,
+                                         &nD);
+                cr.pro += (uint32_t)pro;
+                if (a.tr_after) store_cache_words<V>(cr.cache, lane, N, a.tr_after + unit * NW);
+                if (a.tr_sel && has && (e0 & 31u) == 0u) a.tr_sel[unit * NW + (e0 >> 5)] = csel;
+                if (lane == 0) {
+                    if (a.tr_miss) a.tr_miss[unit] = (uint8_t)nD;
+                    if (a.tr_pro) a.tr_pro[unit] = (uint8_t)pro;
+                }
+            } else {
+                scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R, sel,
+                                         &nD);
+            }
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 cT[v] = nT[v];
@@ -305,7 +332,6 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
                 if (lane * V + v < N) dst[v] = pl[v];
         }
         // store the chain
-        const int NW = (N + 31) >> 5;
         for (int w = 0; w < NW; ++w) {
             const uint32_t contrib = (has && (e0 >> 5) == (uint32_t)w) ? (cr.cache << (e0 & 31)) : 0u;
             const uint32_t wd = __reduce_or_sync(kFull, contrib);

@@ -56,7 +56,8 @@ inline FusedPlan fused_plan(const crc_problem& p, int T) {
 // single-CTA kernel from then on (CRC_EUNSUPPORTED).
 template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR = false>
 int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                   void* state, void* workspace, cudaStream_t stream) {
+                   void* state, void* workspace, const crc_trace* trace,
+                      cudaStream_t stream) {
     using Cfg = FusedCfg<NH, H, PAIR>;
     using RC = typename Cfg::RC;
     const FusedPlan f = fused_plan(p, T);
@@ -133,6 +134,11 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
     a.prog = a.readers + f.ring;
     a.ring_base = ws + f.ctl_bytes;
     a.slot_bytes = f.slot_bytes;
+    a.tr_miss = trace ? trace->misses_dev : nullptr;
+    a.tr_pro = trace ? trace->proactive_dev : nullptr;
+    a.tr_mid = trace ? trace->cache_mid_dev : nullptr;
+    a.tr_after = trace ? trace->cache_after_dev : nullptr;
+    a.tr_sel = trace ? trace->topk_set_dev : nullptr;
     void* args[] = {(void*)&mh, (void*)&mw, (void*)&a};
     cudaError_t e;
     if (PAIR) {
@@ -177,19 +183,20 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
 // when the tiles pair up; CRC_EUNSUPPORTED sends the call to one CTA per tile.
 template <int NH, int H, int V, bool ALL_VALID>
 int launch_fused_pair(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                      void* state, void* workspace, cudaStream_t stream) {
+                      void* state, void* workspace, const crc_trace* trace,
+                      cudaStream_t stream) {
     if constexpr (NH != 128) {
         return CRC_EUNSUPPORTED;
     } else {
         if (p.K <= 2)
             return launch_fused_t<NH, H, V, ALL_VALID, 2, true>(p, hidden, w_cat, T, state,
-                                                                workspace, stream);
+                                                                workspace, trace, stream);
         if (p.K <= 4)
             return launch_fused_t<NH, H, V, ALL_VALID, 4, true>(p, hidden, w_cat, T, state,
-                                                                workspace, stream);
+                                                                workspace, trace, stream);
         if (p.K <= 8)
             return launch_fused_t<NH, H, V, ALL_VALID, 8, true>(p, hidden, w_cat, T, state,
-                                                                workspace, stream);
+                                                                workspace, trace, stream);
         return CRC_EUNSUPPORTED;
     }
 }
@@ -197,22 +204,23 @@ int launch_fused_pair(const crc_problem& p, const uint16_t* hidden, const uint16
 // Dispatch on heads (R > 0 needs the Spatio head) and the Top-K network width.
 template <int NH, int V, bool ALL_VALID>
 int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat,
-                       int T, void* state, void* workspace, cudaStream_t stream) {
+                       int T, void* state, void* workspace, const crc_trace* trace,
+                       cudaStream_t stream) {
 #define CRC_FUSED_KP(HV)                                                                      \
     {                                                                                         \
         const int rc = launch_fused_pair<NH, HV, V, ALL_VALID>(p, hidden, w_cat, T, state,    \
-                                                               workspace, stream);            \
+                                                               workspace, trace, stream);     \
         if (rc != CRC_EUNSUPPORTED) return rc;                                                \
     }                                                                                         \
     if (p.K <= 2)                                                                             \
         return launch_fused_t<NH, HV, V, ALL_VALID, 2>(p, hidden, w_cat, T, state, workspace, \
-                                                       stream);                               \
+                                                       trace, stream);                        \
     if (p.K <= 4)                                                                             \
         return launch_fused_t<NH, HV, V, ALL_VALID, 4>(p, hidden, w_cat, T, state, workspace, \
-                                                       stream);                               \
+                                                       trace, stream);                        \
     if (p.K <= 8)                                                                             \
         return launch_fused_t<NH, HV, V, ALL_VALID, 8>(p, hidden, w_cat, T, state, workspace, \
-                                                       stream);                               \
+                                                       trace, stream);                        \
     return CRC_EUNSUPPORTED;
     if (p.R > 0) {
         CRC_FUSED_KP(3)

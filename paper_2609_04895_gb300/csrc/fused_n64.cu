@@ -4,8 +4,9 @@
 namespace crc {
 
 int launch_fused_n64(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
-                     void* state, void* workspace, cudaStream_t stream) {
-    return launch_fused_for_n<64, 2, true>(p, hidden, w_cat, T, state, workspace, stream);
+                     void* state, void* workspace, const crc_trace* trace,
+                     cudaStream_t stream) {
+    return launch_fused_for_n<64, 2, true>(p, hidden, w_cat, T, state, workspace, trace, stream);
 }
 
 }  // namespace crc

@@ -26,6 +26,7 @@ int launch_policy_t(const crc_problem& p, const float* scores, int T, void* stat
     a.s.trace_pro = trace ? trace->proactive_dev : nullptr;
     a.s.trace_mid = nullptr;                     // cache traces: the method's scan only
     a.s.trace_after = nullptr;
+    a.s.trace_sel = nullptr;
     a.policy = policy;
     a.lambda2 = lambda2;
     const int chains = p.B * p.L;

@@ -283,7 +283,7 @@ def test_full_size_workload(C, oracle_lib, w):
     st = C.State(p)
     tr = C.Trace.alloc(p, w.T)
     C.route_and_cache(p, hd, Wd, st, tr, workspace=ws)
-    fused = st.read(want_caches=True, want_chain_counters=True)
+    fused = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
     assert fused["error"] == 0 and fused["tokens"] == w.T
     cc = fused["chain_counters"]
     assert np.all(cc[..., 0] + cc[..., 1] == w.T * w.K)
@@ -309,20 +309,35 @@ def test_full_size_workload(C, oracle_lib, w):
     C.crc_profile_begin()
     C.route_and_cache(p, hd, Wd, stf, None, workspace=wsf)
     assert C.crc_profile_end()["fused"]["launches"] == 1
-    fz = stf.read(want_caches=True, want_chain_counters=True)
+    fz = stf.read(want_caches=True, want_retention=True, want_chain_counters=True)
     assert fz["error"] == 0 and fz["tokens"] == w.T
     assert np.array_equal(fz["cache_bits"], fused["cache_bits"])
     assert np.array_equal(fz["chain_counters"], fused["chain_counters"])
+    assert np.array_equal(fz["retention"].view(np.uint32), fused["retention"].view(np.uint32))
+    # the same fused kernel writing its per-access trace
+    stt = C.State(p)
+    trf = C.Trace.alloc(p, w.T, caches=True, rank_order=False, topk_set=True)
+    C.crc_profile_begin()
+    C.route_and_cache(p, hd, Wd, stt, trf, workspace=wsf)
+    assert C.crc_profile_end()["fused"]["launches"] == 1
+    ft = stt.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    for k in ("cache_bits", "chain_counters"):
+        assert np.array_equal(ft[k], fz[k]), k
+    assert np.array_equal(ft["retention"].view(np.uint32), fz["retention"].view(np.uint32))
     del wsf
 
-    # fused == pair on every stream
+    # fused == pair on every stream, access by access
     st2 = C.State(p)
-    tr2 = C.Trace.alloc(p, w.T)
+    tr2 = C.Trace.alloc(p, w.T, caches=True, topk_set=True)
     C.cache_scan(p, scores, st2, tr2)
-    pair = st2.read(want_caches=True, want_chain_counters=True)
+    pair = st2.read(want_caches=True, want_retention=True, want_chain_counters=True)
     assert np.array_equal(pair["cache_bits"], fused["cache_bits"])
     assert np.array_equal(pair["chain_counters"], fused["chain_counters"])
+    assert np.array_equal(pair["retention"].view(np.uint32), fused["retention"].view(np.uint32))
     assert torch.equal(tr.topk, tr2.topk) and torch.equal(tr.misses, tr2.misses)
+    for k in ("topk_set", "misses", "proactive", "cache_mid", "cache_after"):
+        assert torch.equal(getattr(trf, k), getattr(tr2, k)), k
+    del trf
 
     # one whole stream: host-generated hidden (same bits), oracle probabilities
     # rounded to fp32 in place of that stream's scores, scan vs the oracle
@@ -362,28 +377,45 @@ FUSED_CASES = [
 
 @pytest.mark.parametrize("name,w", FUSED_CASES, ids=[c[0] for c in FUSED_CASES])
 def test_fused_kernel_equals_pair(C, name, w):
-    """route_and_cache with a workspace large enough for the fused kernel (no
-    trace) equals route_scores + cache_scan bit for bit, over two calls that
-    continue the same streams."""
+    """route_and_cache with a workspace large enough for the fused kernel
+    equals route_scores + cache_scan bit for bit, over two calls that continue
+    the same streams: without a trace, and with the fused kernel writing its
+    per-access trace (Top-K set, misses, proactive loads, the cache after the
+    refinement and after UpdateCache), which must equal the pair's element by
+    element."""
     p = C.problem_of(w)
     W = dev_bf16(S.weights(w, seed=31))
     h = dev_bf16(S.hidden(w, seed=32))
     heads = 3 if w.R > 0 else 2
     split = [w.T // 3, w.T - w.T // 3]
-    st_pair, st_fused = C.State(p), C.State(p)
+    st_pair, st_fused, st_traced = C.State(p), C.State(p), C.State(p)
     ws = torch.empty(C.crc_fused_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    tr_pair, tr_fused = [], []
     t0 = 0
     for n in split:
         hc = h[:, t0:t0 + n].contiguous()
-        C.cache_scan(p, C.route_scores(p, hc, W, heads=heads), st_pair)
+        tp = C.Trace.alloc(p, n, caches=True, topk_set=True)
+        C.cache_scan(p, C.route_scores(p, hc, W, heads=heads), st_pair, tp)
         C.crc_profile_begin()
         C.route_and_cache(p, hc, W, st_fused, None, workspace=ws)
         kt = C.crc_profile_end()
         assert kt["fused"]["launches"] == 1 and kt["router"]["launches"] == 0
+        tf = C.Trace.alloc(p, n, caches=True, rank_order=False, topk_set=True)
+        C.crc_profile_begin()
+        C.route_and_cache(p, hc, W, st_traced, tf, workspace=ws)
+        kt = C.crc_profile_end()
+        assert kt["fused"]["launches"] == 1 and kt["router"]["launches"] == 0
+        tr_pair.append(tp)
+        tr_fused.append(tf)
         t0 += n
     a = st_pair.read(want_caches=True, want_retention=True, want_chain_counters=True)
-    b = st_fused.read(want_caches=True, want_retention=True, want_chain_counters=True)
-    assert b["error"] == 0 and b["tokens"] == w.T
-    for k in ("cache_bits", "chain_counters"):
-        assert np.array_equal(a[k], b[k]), k
-    assert np.array_equal(a["retention"].view(np.uint32), b["retention"].view(np.uint32))
+    for st in (st_fused, st_traced):
+        b = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
+        assert b["error"] == 0 and b["tokens"] == w.T
+        for k in ("cache_bits", "chain_counters"):
+            assert np.array_equal(a[k], b[k]), k
+        assert np.array_equal(a["retention"].view(np.uint32), b["retention"].view(np.uint32))
+    for k in ("topk_set", "misses", "proactive", "cache_mid", "cache_after"):
+        g = torch.cat([getattr(x, k) for x in tr_fused], dim=1)
+        r = torch.cat([getattr(x, k) for x in tr_pair], dim=1)
+        assert torch.equal(g, r), k

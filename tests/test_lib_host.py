@@ -39,7 +39,7 @@ def test_every_declared_symbol_is_exported_and_bound(crc):
 
 def test_struct_layouts_match_header(crc):
     assert ctypes.sizeof(crc.crc_problem) == 40
-    assert ctypes.sizeof(crc.crc_trace) == 40
+    assert ctypes.sizeof(crc.crc_trace) == 48
     assert ctypes.sizeof(crc.crc_transfer) == 24
     assert ctypes.sizeof(crc.crc_stats) == 56
 
