@@ -105,11 +105,12 @@ typedef struct crc_stats {
 
 /* ------------------------------------------------------------------------ */
 /* State: a caller-owned device buffer holding, per (stream, layer), the    */
-/* cache set C_{t,l} (bitmask), the carried retention score s^T_{t-1,l}     */
-/* (= a^T_{t,l}, fp32 [N]) and hit / miss / proactive counters; per stream  */
-/* the carried Spatio prediction p^S_{t-1,L-1} (the wrap-around             */
-/* predecessor of layer 0); and the next token index.  Successive calls on  */
-/* one state continue the same streams: processing T tokens in chunks gives */
+/* cache set C_{t,l} that Algorithms 1 and 2 update (bitmask), the carried  */
+/* retention score s^T_{t-1,l} (= a^T_{t,l} of Sec. 3.3, fp32 [N]) and the  */
+/* hit / miss / proactive counters of Sec. 4.1; per stream the carried      */
+/* Spatio prediction p^S_{t-1,L-1} (the wrap-around causal predecessor of   */
+/* layer 0, Sec. 3.3); and the next token index.  Successive calls on one   */
+/* state continue the same streams: processing T tokens in chunks gives     */
 /* bit-identical results to one call.  Two calls on one state must not run  */
 /* concurrently.                                                            */
 /* ------------------------------------------------------------------------ */
@@ -117,18 +118,45 @@ typedef struct crc_stats {
 /* Bytes needed for the state of problem p (0 if p is invalid). */
 size_t crc_state_bytes(const crc_problem *p);
 
-/* Cold start: empty caches, zero counters, token 0.  state_dev must be
- * 256-byte aligned and hold crc_state_bytes(p) bytes.  Asynchronous. */
+/* Cold start: empty caches (the not-full branches of Algorithms 1 and 2
+ * fill them), zero counters, token 0.  state_dev must be 256-byte aligned and
+ * hold crc_state_bytes(p) bytes.  Asynchronous. */
 int crc_state_init(const crc_problem *p, void *state_dev, size_t state_bytes, void *stream);
 
-/* Synchronises `stream`, then reads the state back: totals into *out
- * (required); optionally cache bitmasks [B][L][ceil(N/32)] (bit e % 32 of
+/* Synchronises `stream`, then reads the state back: the Sec. 4.1 totals
+ * into *out (required); optionally cache bitmasks [B][L][ceil(N/32)] (bit e % 32 of
  * word e / 32 set when expert e is resident), the carried retention scores
  * [B][L][N] and per-(stream, layer) counters [B][L][3] = hits, misses,
  * proactive.  Returns the latched device error if there is one. */
 int crc_state_read(const crc_problem *p, const void *state_dev, size_t state_bytes,
                    crc_stats *out, uint32_t *cache_bits_host, float *retention_host,
                    uint64_t *chain_counters_host, void *stream);
+
+/* The paper's reported metrics (Sec. 4.1 Metrics) from the totals of
+ * crc_state_read, over all B streams: with A accesses, D demand misses, P
+ * proactive loads, S_exp = expert_bytes and B * tokens decode tokens,
+ *   hit                  = 1 - D / A             (NaN when A = 0)
+ *   adj_hit              = (A - D) / (A + P)     (NaN when A + P = 0)
+ *   traffic_bytes        = (D + P) * S_exp
+ *   load_per_token_bytes = (D + P) * S_exp / (B * tokens)   (0 with no token)
+ * Host-only arithmetic; CRC_EINVAL for a null pointer or invalid problem. */
+typedef struct crc_report {
+    double hit;
+    double adj_hit;
+    double traffic_bytes;
+    double load_per_token_bytes;
+} crc_report;
+int crc_metrics(const crc_problem *p, const crc_stats *s, crc_report *out);
+
+/* Exposed expert-loading cost per decode token under the overlap model of
+ * the paper's appendix on asynchronous transfer overlap: each expert
+ * transfer takes c_exp seconds, demand transfers are fully exposed and a
+ * fraction eta of the proactive ones is hidden behind computation,
+ *   *t_load = c_exp / (B * tokens) * (D + (1 - eta) * P)   (0 with no token).
+ * Host-only; CRC_EINVAL for a null pointer, an invalid problem, eta outside
+ * [0, 1] or a negative or non-finite c_exp. */
+int crc_load_time(const crc_problem *p, const crc_stats *s, double c_exp, double eta,
+                  double *t_load);
 
 /* ------------------------------------------------------------------------ */
 /* Hot path                                                                 */
@@ -199,8 +227,11 @@ size_t crc_workspace_bytes(const crc_problem *p, int32_t chunk_tokens);
  * smaller workspaces, take the chunked two-kernel path.  0 if p is invalid. */
 size_t crc_fused_workspace_bytes(const crc_problem *p);
 
-/* The whole step: router heads and cache simulation over T tokens, the
- * same results as crc_route_scores followed by crc_cache_scan (bit for bit).
+/* The whole step of the paper's decoding loop over T tokens: the router
+ * heads (Sec. 2, 3.2, 3.3), then per access the pre-access refinement and
+ * access of Algorithm 2 with UpdateCache (Algorithm 1) and the Sec. 4.1
+ * accounting -- the same results as crc_route_scores followed by
+ * crc_cache_scan (bit for bit).
  * hidden_dev bf16 [B][T][L][d]; w_cat_dev bf16 [L][3N][d] (the S head is
  * not computed when R = 0).  The router scores never leave the workspace.
  * With workspace_bytes >= crc_fused_workspace_bytes(p), K <= 8 and a trace
@@ -293,20 +324,28 @@ int crc_wait_probe(const crc_problem *p, void *state_dev, size_t state_bytes, in
  * initialisation (cudaMalloc / cudaFree may also synchronise the whole
  * device, which a latency-bound decode loop cannot afford).  The caller still
  * provides every input and output (hidden states, weights, state, trace).
- * This call allocates nothing: the router scores of each chunk of tokens go
- * to a fixed array compiled into the library, CRC_NOALLOC_SCRATCH_BYTES bytes
- * on every GPU where the library is loaded, kept until the process exits.
- * The chunk is the largest number of tokens whose scores fit in it; a problem
- * whose scores for one token do not fit (B * L * 3N * 4 bytes above
- * CRC_NOALLOC_SCRATCH_BYTES) is refused with CRC_EUNSUPPORTED before anything
- * is enqueued.  The first call on a device looks up that device's copy of the
- * array (once per device, with the device current); make that first call
- * before any stream capture.  All calls share the one array per device and
- * it keeps the last call's contents (nothing in it needs to start at zero:
- * each chunk's scores are written in full before they are read), so calls
- * whose kernels may overlap on the GPU -- unordered streams or concurrent
- * host threads -- race on it: order them.  Results are bit-identical to
- * crc_route_and_cache. */
+ * This call allocates nothing: its scratch is a fixed array compiled into the
+ * library, CRC_NOALLOC_SCRATCH_BYTES bytes on every GPU where the library is
+ * loaded, kept until the process exits.  The array takes one of two layouts,
+ * exactly as a caller workspace of that size would in crc_route_and_cache:
+ *  - when crc_fused_workspace_bytes(p) <= CRC_NOALLOC_SCRATCH_BYTES (small
+ *    problems: few streams and layers) and the trace, if any, leaves topk_dev
+ *    NULL, the call is the fused kernel, with its control words and its ring
+ *    of router-score tiles in the array (the control words are cleared by the
+ *    call itself before the kernel starts);
+ *  - otherwise the router scores of each chunk of tokens go to the array, the
+ *    chunk being the largest number of tokens whose scores (B * L * 3N * 4
+ *    bytes per token) fit in it; a problem whose scores for one token do not
+ *    fit is refused with CRC_EUNSUPPORTED before anything is enqueued.
+ * The first call on a device looks up that device's copy of the array (once
+ * per device, with the device current); make that first call before any
+ * stream capture.  The address is kept for the life of the process, so a
+ * device reset (cudaDeviceReset) after that first call is not supported.
+ * All calls share the one array per device and it keeps the last call's
+ * contents (nothing in it needs to start at zero beyond what each call
+ * clears itself), so calls whose kernels may overlap on the GPU -- unordered
+ * streams or concurrent host threads -- race on it: order them.  Results are
+ * bit-identical to crc_route_and_cache. */
 int crc_route_and_cache_noalloc(const crc_problem *p, const uint16_t *hidden_dev,
                                 const uint16_t *w_cat_dev, int32_t T, void *state_dev,
                                 size_t state_bytes, const crc_trace *trace, void *stream);

@@ -52,6 +52,11 @@ class crc_stats(ctypes.Structure):
                 ("error", ctypes.c_uint32), ("reserved", ctypes.c_uint32)]
 
 
+class crc_report(ctypes.Structure):
+    _fields_ = [("hit", ctypes.c_double), ("adj_hit", ctypes.c_double),
+                ("traffic_bytes", ctypes.c_double), ("load_per_token_bytes", ctypes.c_double)]
+
+
 KERNEL_KINDS = {"router": 0, "scan": 1, "state": 2, "synth": 3, "fused": 4, "loss": 5,
                 "loss_means": 6}
 
@@ -98,6 +103,9 @@ EXPORTS = [
     ("crc_transfer_plan", ctypes.c_int, [PP, I32, P, P, P, P, P, ctypes.c_int64, P]),
     ("crc_transfer_replay", ctypes.c_int, [PP, P, ctypes.c_int64, P, ctypes.c_int64, P, P]),
     ("crc_cache_loss", ctypes.c_int, [PP, P, I32, I32, I32, D, D, D, P, P, P, P, SZ, P]),
+    ("crc_metrics", ctypes.c_int, [PP, ctypes.POINTER(crc_stats), ctypes.POINTER(crc_report)]),
+    ("crc_load_time", ctypes.c_int, [PP, ctypes.POINTER(crc_stats), D, D,
+                                      ctypes.POINTER(ctypes.c_double)]),
     ("crc_launch_count", U64, []),
     ("crc_strerror", ctypes.c_char_p, [ctypes.c_int]),
     ("crc_profile_begin", ctypes.c_int, []),
@@ -538,28 +546,31 @@ def synth_hidden(B, T, L, d, seed=0, rho_t=0.9, rho_l=0.8, t0=0, carry=None, att
     return out, carry
 
 
+def _stats_struct(stats: dict) -> crc_stats:
+    st = crc_stats()
+    for f, _ in crc_stats._fields_:
+        if f in stats and f != "reserved":
+            setattr(st, f, int(stats[f]))
+    return st
+
+
 def load_time(stats: dict, p: crc_problem, c_exp: float, eta: float) -> float:
-    """Exposed expert-loading cost per decode token under the paper's overlap
-    model (appendix on asynchronous transfer overlap): every expert transfer
-    takes c_exp seconds, demand transfers are fully exposed and a fraction eta
-    of the proactive ones is hidden by computation:
-    t_load(eta) = c_exp / T * (D + (1 - eta) * P), T = decode tokens."""
+    """crc_load_time: exposed expert-loading cost per decode token under the
+    paper's overlap model, from the totals of crc_state_read (a dict as
+    returned by State.read)."""
     if not 0.0 <= eta <= 1.0:
         raise ValueError("eta must lie in [0, 1]")
-    tokens = stats["tokens"] * p.B
-    if tokens == 0:
-        return 0.0
-    return c_exp / tokens * (stats["misses"] + (1.0 - eta) * stats["proactive"])
+    out = ctypes.c_double()
+    _ck(load().crc_load_time(ctypes.byref(p), ctypes.byref(_stats_struct(stats)), c_exp, eta,
+                             ctypes.byref(out)), "crc_load_time")
+    return out.value
 
 
 def metrics(stats: dict, p: crc_problem) -> dict:
-    """Hit, AdjHit and Load/token (bytes per decode token) of Sec. 4.1 from
-    the totals of crc_state_read; decode tokens = streams x tokens per stream."""
-    A, D, Pn = stats["accesses"], stats["misses"], stats["proactive"]
-    tokens = stats["tokens"] * p.B
-    return {
-        "hit": 1.0 - D / A if A else float("nan"),
-        "adj_hit": (A - D) / (A + Pn) if A + Pn else float("nan"),
-        "traffic_bytes": (D + Pn) * p.expert_bytes,
-        "load_per_token_bytes": (D + Pn) * p.expert_bytes / tokens if tokens else 0.0,
-    }
+    """crc_metrics: Hit, AdjHit, traffic and Load/token (bytes per decode
+    token) of Sec. 4.1 from the totals of crc_state_read."""
+    r = crc_report()
+    _ck(load().crc_metrics(ctypes.byref(p), ctypes.byref(_stats_struct(stats)), ctypes.byref(r)),
+        "crc_metrics")
+    return {"hit": r.hit, "adj_hit": r.adj_hit, "traffic_bytes": r.traffic_bytes,
+            "load_per_token_bytes": r.load_per_token_bytes}

@@ -176,6 +176,30 @@ int crc_state_read(const crc_problem* p, const void* state_dev, size_t state_byt
     return h.error ? (int)h.error : CRC_OK;
 }
 
+int crc_metrics(const crc_problem* p, const crc_stats* s, crc_report* out) {
+    if (!s || !out || check_problem(p, false) != CRC_OK) return CRC_EINVAL;
+    const double A = (double)s->accesses, D = (double)s->misses, P = (double)s->proactive;
+    const double tokens = (double)p->B * (double)s->tokens;
+    const double moved = (D + P) * (double)p->expert_bytes;
+    out->hit = A > 0.0 ? 1.0 - D / A : NAN;
+    out->adj_hit = A + P > 0.0 ? (A - D) / (A + P) : NAN;
+    out->traffic_bytes = moved;
+    out->load_per_token_bytes = tokens > 0.0 ? moved / tokens : 0.0;
+    return CRC_OK;
+}
+
+int crc_load_time(const crc_problem* p, const crc_stats* s, double c_exp, double eta,
+                  double* t_load) {
+    if (!s || !t_load || check_problem(p, false) != CRC_OK) return CRC_EINVAL;
+    if (!(eta >= 0.0 && eta <= 1.0) || !(c_exp >= 0.0) || !std::isfinite(c_exp))
+        return CRC_EINVAL;
+    const double tokens = (double)p->B * (double)s->tokens;
+    *t_load = tokens > 0.0
+                  ? c_exp / tokens * ((double)s->misses + (1.0 - eta) * (double)s->proactive)
+                  : 0.0;
+    return CRC_OK;
+}
+
 int crc_route_scores(const crc_problem* p, const uint16_t* hidden_dev, const uint16_t* w_cat_dev,
                      int32_t T, int32_t heads, float* scores_dev, void* stream) {
     int rc = check_problem(p, true);

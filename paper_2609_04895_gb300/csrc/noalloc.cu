@@ -18,6 +18,8 @@ std::vector<void*> g_scratch_ptr;   // device address of the array, per device
 // Device address of this device's copy of the array.  In host code the
 // array's name only stands for the symbol; handing it to a kernel would use
 // the wrong memory, so the address is looked up with the device current.
+// It is kept for the life of the process: a device reset after the first call
+// would leave it stale, which is why the entry point does not support one.
 int scratch_for_current_device(void** out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return CRC_ECUDA;

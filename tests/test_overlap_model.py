@@ -77,3 +77,27 @@ def test_product_function_matches_the_oracle(oracle_lib):
             oracle_lib.load_time(37, 11, 25 * 3, 2e-3, eta), rel=1e-15)
     with pytest.raises(ValueError):
         crc.load_time(stats, p, 1.0, 1.5)
+
+
+def test_product_metrics_match_the_oracle(oracle_lib):
+    # crc_metrics (the C ABI) against the oracle's Sec. 4.1 metric function
+    from paper_2609_04895_gb300 import crc
+    p = crc.problem(L=48, N=128, K=8, d=2048, C=32, R=4, B=5, expert_bytes=3 * 2048 * 768 * 2)
+    rng = np.random.default_rng(9)
+    for _ in range(50):
+        tokens = int(rng.integers(1, 5000))
+        A = p.L * p.K * tokens * p.B
+        D = int(rng.integers(0, A + 1))
+        P = int(rng.integers(0, 3 * A))
+        stats = {"accesses": A, "hits": A - D, "misses": D, "proactive": P, "tokens": tokens}
+        m = crc.metrics(stats, p)
+        o = oracle_lib.metrics(A, D, P, tokens * p.B, p.expert_bytes)
+        assert m["hit"] == pytest.approx(o["hit"], rel=1e-15, abs=1e-15)
+        assert m["adj_hit"] == pytest.approx(o["adj_hit"], rel=1e-15, abs=1e-15)
+        assert m["load_per_token_bytes"] == pytest.approx(o["load_per_token"], rel=1e-15)
+        assert m["traffic_bytes"] == (D + P) * p.expert_bytes
+    empty = crc.metrics({"accesses": 0, "misses": 0, "proactive": 0, "tokens": 0}, p)
+    assert np.isnan(empty["hit"]) and np.isnan(empty["adj_hit"])
+    assert empty["load_per_token_bytes"] == 0.0
+    with pytest.raises(crc.CrcError):
+        crc.load_time({"misses": 1, "proactive": 1, "tokens": 1}, p, -1.0, 0.5)

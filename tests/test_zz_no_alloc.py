@@ -5,8 +5,10 @@ serving framework that owns all device memory through its own pool, a
 plug-in whose host forbids allocation after start-up): instead of a caller
 workspace it uses a scratch array compiled into the library.  These tests
 call it through the C ABI and check that two calls in a row, on different
-inputs, give exactly what crc_route_and_cache gives, and that a problem too
-large for the array is refused.  The file sorts last so that a run stopping
+inputs, give exactly what crc_route_and_cache gives -- in both layouts of the
+array (the per-chunk router scores of the two-kernel path, and the fused
+kernel's control words and ring of tiles) -- and that a problem too large for
+the array is refused.  The file sorts last so that a run stopping
 at its first failure has already run every other test.
 """
 import ctypes
@@ -62,6 +64,39 @@ def test_noalloc_matches_route_and_cache_on_two_calls_in_a_row(C):
         assert torch.equal(tgot.topk, tref.topk), call
         assert torch.equal(tgot.misses, tref.misses), call
         assert torch.equal(tgot.proactive, tref.proactive), call
+
+
+def test_noalloc_fused_kernel_in_the_scratch_on_two_calls_in_a_row(C):
+    # A problem small enough for the fused kernel's ring to fit the array: an
+    # untraced call (and one whose trace leaves out the rank-order Top-K) runs
+    # the fused kernel with its control words and ring in the shared array.
+    # Two calls in a row on different inputs, each against crc_route_and_cache
+    # with a workspace of its own.
+    w = S.QWEN3_30B.with_(B=8, L=6, T=300)
+    p = C.problem_of(w)
+    assert 0 < C.crc_fused_workspace_bytes(p) <= C.NOALLOC_SCRATCH_BYTES
+    W = C.synth_weights(w.L, w.N, w.d, seed=4)
+    ws = torch.empty(C.crc_fused_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    for call, seed in enumerate((23, 24)):
+        h, _ = C.synth_hidden(w.B, w.T, w.L, w.d, seed=seed, rho_t=w.rho_t, rho_l=w.rho_l)
+        ref_st = C.State(p)
+        C.crc_route_and_cache(p, h.data_ptr(), W.data_ptr(), w.T, ref_st.ptr, ref_st.nbytes,
+                              None, ws.data_ptr(), ws.numel())
+        ref = ref_st.read(want_caches=True, want_retention=True, want_chain_counters=True)
+        for traced in (False, True):
+            st = C.State(p)
+            tr = C.Trace.alloc(p, w.T, rank_order=False, topk_set=True) if traced else None
+            C.crc_profile_begin()
+            C.crc_route_and_cache_noalloc(p, h.data_ptr(), W.data_ptr(), w.T, st.ptr, st.nbytes,
+                                          None if tr is None else tr.c())
+            kt = C.crc_profile_end()
+            assert kt["fused"]["launches"] == 1 and kt["router"]["launches"] == 0, (call, traced)
+            got = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
+            assert got["error"] == 0 and got["tokens"] == w.T, (call, traced)
+            for k in ("cache_bits", "chain_counters"):
+                assert np.array_equal(got[k], ref[k]), (call, traced, k)
+            assert np.array_equal(got["retention"].view(np.uint32),
+                                  ref["retention"].view(np.uint32)), (call, traced)
 
 
 def test_noalloc_refuses_problems_larger_than_its_scratch(C):
