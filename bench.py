@@ -608,21 +608,24 @@ def run_reference(args):
     oracle.build()
     threads = oracle.default_threads()
     Wb = S.weights(w, seed=0)
-    # size one step at a few seconds of oracle time
-    h1 = S.hidden(w.with_(B=1), seed=0, T=min(4, w.T))
+    # one stream per host core (the oracle's scan runs a thread per stream,
+    # its router heads a thread per core), as many tokens as make one step a
+    # few seconds of oracle time
+    ns = max(1, min(w.B, threads))
+    h1 = S.hidden(w, seed=0, streams=range(ns), T=min(4, w.T))
     t0 = time.perf_counter()
     oracle.run(h1, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
-    rate = h1.shape[1] * w.L / max(time.perf_counter() - t0, 1e-6)
+    rate = ns * h1.shape[1] * w.L / max(time.perf_counter() - t0, 1e-6)
     budget = max(1.0, min(6.0, 150.0 / max(1, args.steps + args.warmup)))
-    nt = int(min(w.T, max(4, rate * budget // w.L)))
-    h = S.hidden(w.with_(B=1), seed=0, T=nt)
+    nt = int(min(w.T, max(4, rate * budget // (ns * w.L))))
+    h = S.hidden(w, seed=0, streams=range(ns), T=nt)
     for _ in range(args.warmup):
         oracle.run(h, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
     t0 = time.perf_counter()
     for _ in range(args.steps):
         oracle.run(h, Wb, w.N, w.K, w.C, w.R, margins=False, nthreads=threads)
     dt = time.perf_counter() - t0
-    units = nt * w.L
+    units = ns * nt * w.L
     value = units * args.steps / dt
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
@@ -630,8 +633,9 @@ def run_reference(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": workload_config(w), "impl": "reference",
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                         "sample": f"1 stream x {nt} tokens x {w.L} layers = {units} decisions "
-                                   f"per step (fp64 router heads + literal scan)"},
+                         "sample": f"{ns} stream(s) x {nt} tokens x {w.L} layers = {units} "
+                                   f"decisions per step of the workload named in config "
+                                   f"(fp64 router heads + literal scan)"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)

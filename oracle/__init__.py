@@ -12,8 +12,9 @@ caches and score orders, the closed forms of Algorithms 1 and 2 on a full
 cache, the special cases C = K (R = 0), C = N, constant hidden state, R = 0
 equals update-only, copy-initialised heads, a library softmax cross-check,
 the published Philox test vectors for the input generator, hand-traced
-worked examples under ``tests/golden/`` and the paper's printed metric
-identities (Table 1, Table 2).
+worked examples (``tests/test_oracle_scan.py``), hand-built accesses whose
+closest decision is known (``tests/test_oracle_margins.py``) and the paper's
+printed metric identities (Table 1, Table 2; ``tests/golden/``).
 """
 from __future__ import annotations
 

@@ -494,7 +494,8 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
     const int64_t t0 = hdr->t_next;
     const uint32_t parity = hdr->parity;
 
-    if (active && hdr_ok) {
+    uint32_t* err = &hdr->error;
+    if (active && hdr_ok && CRC_IN_BOUNDS(a.trace_t0 >= 0 && a.trace_t0 + a.T <= a.trace_T, err)) {
         const int b = chain / a.L, l = chain % a.L;
         const int N = a.N, L = a.L, T = a.T;
         const size_t row = (size_t)3 * N;
@@ -516,6 +517,10 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
         cr.hits = cr.misses = cr.pro = 0u;
 
         const float* base = a.scores + lane * V;
+        // debug builds: the unit a pointer is formed for lies inside scores [B][T][L]
+        auto unit_ok = [&](int t, int ll) {
+            return CRC_IN_BOUNDS(b < a.B && t >= 0 && t < T && ll >= 0 && ll < L, err);
+        };
         auto unit_ptr = [&](int t, int ll) -> const float* {
             return base + (((size_t)b * T + t) * L + ll) * row;
         };
@@ -533,13 +538,14 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
         uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) & 3];
         const float* row_base = a.scores + ((size_t)b * T * L + l) * row;   // token 0 of chain
 
-        Vec<V> cR = load_vec<V>(unit_ptr(0, l), has);
-        Vec<V> cT = load_vec<V>(unit_ptr(0, l) + N, has);
-        Vec<V> cS = load_vec<V>(pred_ptr(0), has && want_s && (t0 + 0 >= 1));
+        Vec<V> cR = load_vec<V>(unit_ptr(0, l), has && unit_ok(0, l));
+        Vec<V> cT = load_vec<V>(unit_ptr(0, l) + N, has && unit_ok(0, l));
+        Vec<V> cS = load_vec<V>(pred_ptr(0), has && want_s && (t0 + 0 >= 1) &&
+                                                 (l > 0 ? unit_ok(0, l - 1) : true));
         for (int t = 0; t < T; ++t) {
             if (batch_sel && (t & 31) == 0) {
                 __syncwarp();
-                if (t + lane < T) {
+                if (t + lane < T && unit_ok(t + lane, l)) {
                     const float* r = row_base + (size_t)(t + lane) * L * row;
                     row_topk_mask<KP>(r, N, a.K, sel_rows[lane]);
                 }
@@ -548,13 +554,16 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
             uint32_t sel_in = 0u;
             if (batch_sel && has) {
                 const uint32_t e0 = (uint32_t)lane * V;
-                sel_in = (sel_rows[t & 31][e0 >> 5] >> (e0 & 31)) & ((1u << V) - 1u);
+                if (CRC_IN_BOUNDS((e0 >> 5) < 8u, err))
+                    sel_in = (sel_rows[t & 31][e0 >> 5] >> (e0 & 31)) & ((1u << V) - 1u);
             }
             Vec<V> nR, nT, nS;
             if (t + 1 < T) {
-                nR = load_vec<V>(unit_ptr(t + 1, l), has);
-                nT = load_vec<V>(unit_ptr(t + 1, l) + N, has);
-                nS = load_vec<V>(pred_ptr(t + 1), has && want_s);
+                const bool ok1 = unit_ok(t + 1, l);
+                nR = load_vec<V>(unit_ptr(t + 1, l), has && ok1);
+                nT = load_vec<V>(unit_ptr(t + 1, l) + N, has && ok1);
+                nS = load_vec<V>(pred_ptr(t + 1), has && want_s &&
+                                                      (l > 0 ? unit_ok(t + 1, l - 1) : unit_ok(t, L - 1)));
             }
             const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
             scan_step<V, ALL_VALID>(cr, cR.v, cT.v, cS.v, want_s && (t0 + t >= 1), valid, lane, a.K, a.C,
@@ -564,6 +573,9 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
                          a.trace_mid ? a.trace_mid + unit * (size_t)((N + 31) >> 5) : nullptr,
                          a.trace_after ? a.trace_after + unit * (size_t)((N + 31) >> 5) : nullptr,
                          N, a.trace_sel ? a.trace_sel + unit * (size_t)((N + 31) >> 5) : nullptr);
+            // debug builds: every expert the step made resident lies in this
+            // lane's range and the cache holds at most C experts
+            (void)CRC_IN_BOUNDS((cr.cache & ~valid) == 0u && cr.count <= a.C, err);
             cR = nR;
             cT = nT;
             cS = nS;
@@ -577,7 +589,7 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
             const uint32_t word = __reduce_or_sync(kFull, contrib);
             if (lane == 0) cs.bits[w] = word;
         }
-        if (has) {
+        if (has && CRC_IN_BOUNDS(chain < a.B * a.L, err)) {
 #pragma unroll
             for (int v = 0; v < V; ++v)
                 if (lane * V + v < N) retention[(size_t)chain * N + lane * V + v] = cr.aT[v];

@@ -61,6 +61,23 @@ __device__ __forceinline__ void latch_error(uint32_t* word, uint32_t code) {
     if (word) atomicCAS(word, 0u, code);
 }
 
+// Debug builds (compiled with -DCRC_DEBUG) check every index a kernel derives
+// before it addresses memory with it -- streams, layers, chains, tokens, ring
+// slots and tile rows, experts -- against the bound of the array it indexes.
+// A failed check latches CRC_EDEVICE in the error word and the access is
+// skipped (a skipped load leaves its default), so a wrong index surfaces as an
+// error code the host reads, never as a stray access.  Release builds compile
+// every check to `true`.
+__device__ __forceinline__ bool dbg_check(bool ok, uint32_t* err) {
+    if (!ok) latch_error(err, CRC_EDEVICE);
+    return ok;
+}
+#ifdef CRC_DEBUG
+#define CRC_IN_BOUNDS(cond, err) ::crc::dbg_check((cond), (err))
+#else
+#define CRC_IN_BOUNDS(cond, err) true
+#endif
+
 // ---------------------------------------------------------------------------
 // generic helpers
 // ---------------------------------------------------------------------------

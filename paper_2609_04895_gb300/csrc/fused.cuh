@@ -207,6 +207,12 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
         const int k_ps = (tb * L + (l > 0 ? l - 1 : L - 1)) * a.n_bg + bg;
         const int k_prev = (l == 0 && tb > 0) ? ((tb - 1) * L + L - 1) * a.n_bg + bg : -1;
         const bool read_ps = want_s && (l > 0 || a.TB >= 2);
+        // debug builds: the item's stream, layer, block, tiles and rows exist
+        if (!CRC_IN_BOUNDS(b < a.B && l < L && tb < a.n_tb && k_own < a.num_tiles &&
+                               k_ps < a.num_tiles && k_prev < a.num_tiles &&
+                               sbi * a.TB + a.TB <= 128 && parity < 2u,
+                           err))
+            break;
         // wait for the chain's previous block and the tiles this item reads
         bool ok = true;
         if (lane == 0) {
@@ -296,7 +302,7 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
             const bool refine = want_s && tbi >= refine_from;
             const uint32_t sel = (csel >> (e0 & 31)) & ((1u << V) - 1u);
             int nD;
-            if (traced) {
+            if (traced && CRC_IN_BOUNDS(tb * a.TB + tbi < a.T, err)) {
                 // the refinement on its own, so the cache between the phases is seen
                 const size_t unit = ((size_t)b * a.T + tb * a.TB + tbi) * L + l;
                 const int pro = refine ? scan_refine<V, ALL_VALID>(cr, cS, valid, lane, a.C, a.R)
@@ -315,6 +321,9 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
                 scan_apply<V, ALL_VALID>(cr, cT, cS, refine, valid, lane, a.K, a.C, a.R, sel,
                                          &nD);
             }
+            // debug builds: every expert the step made resident lies in this
+            // lane's range and the cache holds at most C experts
+            (void)CRC_IN_BOUNDS((cr.cache & ~valid) == 0u && cr.count <= a.C, err);
 #pragma unroll
             for (int v = 0; v < V; ++v) {
                 cT[v] = nT[v];
@@ -644,8 +653,8 @@ __global__ void __launch_bounds__(512, 1)
             const int slot = k % a.ring;
             const uint32_t gen = (uint32_t)(k / a.ring);
             // the slot's previous tile must be fully read
-            bool ok = true;
-            if (lane == 0 && gen > 0)
+            bool ok = CRC_IN_BOUNDS(slot < a.ring && l < a.L && bg < a.n_bg && tb < a.n_tb, err);
+            if (lane == 0 && gen > 0 && ok)
                 ok = wait_geq(&a.readers[slot], target_per_tile * gen, abort_flag, err);
             ok = __shfl_sync(kFull, ok, 0);
             uint8_t* slot_p = a.ring_base + (size_t)slot * a.slot_bytes;
