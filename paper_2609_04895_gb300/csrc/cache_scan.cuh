@@ -42,6 +42,8 @@ struct ScanArgs {
 // empty slot.  Each lane keeps (key, slot) pairs sorted in policy order
 // (key descending, equal keys by ascending slot = ascending expert index).
 __device__ __forceinline__ uint32_t pkey(float x) { return __float_as_uint(x) + 1u; }
+__device__ __forceinline__ uint32_t umin(uint32_t a, uint32_t b) { return a < b ? a : b; }
+__device__ __forceinline__ uint32_t umax(uint32_t a, uint32_t b) { return a > b ? a : b; }
 
 template <int V>
 struct KeyList {
@@ -93,25 +95,25 @@ __device__ __forceinline__ int warp_pop_first(KeyList<V>& L, int lane, uint32_t&
 
 // Last member in policy order among the slots flagged in `members`: smallest
 // key and, among equal keys, the highest index.  Returns the owner lane (-1 if
-// no member); the owner receives the slot.
+// no member); the owner receives the slot.  Keys are >= 1, so a non-member
+// counts as the largest key, 0xffffffff, which no real key reaches.
 template <int V>
 __device__ __forceinline__ int warp_last_member(const uint32_t (&k)[V], uint32_t members,
                                                 int lane, uint32_t& key, uint32_t& slot) {
-    uint32_t best = 0xffffffffu, bs = 0u;
-    bool has = false;
+    uint32_t m[V];
 #pragma unroll
-    for (int v = 0; v < V; ++v) {
-        if (((members >> v) & 1u) && k[v] <= best) {
-            best = k[v];
-            bs = v;
-            has = true;
-        }
-    }
-    const uint32_t mn = __reduce_min_sync(kFull, has ? best : 0xffffffffu);
+    for (int v = 0; v < V; ++v) m[v] = ((members >> v) & 1u) ? k[v] : 0xffffffffu;
+    uint32_t best = m[0];
+#pragma unroll
+    for (int v = 1; v < V; ++v) best = umin(best, m[v]);
+    const uint32_t mn = __reduce_min_sync(kFull, best);
     key = mn;
-    const uint32_t b = __ballot_sync(kFull, has && best == mn);
-    if (b == 0u) return -1;
+    const uint32_t b = __ballot_sync(kFull, best == mn);
+    if (mn == 0xffffffffu) return -1;
     const int owner = 31 - __clz(b);
+    uint32_t bs = 0u;
+#pragma unroll
+    for (int v = 0; v < V; ++v) bs = m[v] == mn ? (uint32_t)v : bs;   // the highest such slot
     if (lane == owner) slot = bs;
     return owner;
 }
@@ -295,69 +297,96 @@ __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, ui
     }
 }
 
-// Refinement, access and UpdateCache of one access, given s^T = p^R + p^T,
-// the Spatio prediction of the predecessor and the native Top-K set `sel`
-// (this lane's V bits).  Updates the chain registers; returns the number of
-// proactive loads and writes the demand misses to *n_miss.
 // Algorithm 2's pre-access refinement of the chain's cache with priorities
 // a[e] + pS[e] (s^ST for the method, s^S for the Spatio-only ablation): the
-// top-R candidates in order, each skipped when resident, loaded into a free
-// slot, or swapped for the lowest resident when strictly higher.  Returns the
-// proactive loads.
+// candidates A = Top_R of all experts in descending order, each skipped when
+// resident, loaded into a free slot, or swapped for the lowest resident when
+// strictly higher.  Returns the proactive loads.
+//
+// Only the non-resident members of A can change the cache, so they are taken
+// one at a time in order -- the best remaining non-resident c -- and c is a
+// member of A exactly when fewer than R experts precede it in the order: the j
+// non-residents already loaded and the residents of the original cache ahead
+// of it.  The first such count is also the test that leaves the cache alone
+// when at least R residents precede every non-resident.  An original resident
+// that a candidate evicted is never taken as a candidate itself: in the
+// literal loop it would meet a cache whose lowest member is no lower than it
+// and lose the strict test, ending the pass exactly as the rank test or the
+// strict test ends it here.
 template <int V, bool ALL_VALID>
 __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V], uint32_t valid,
                                            int lane, int C, int R) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
+    uint32_t kS[V];
+#pragma unroll
+    for (int v = 0; v < V; ++v)
+        kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;
+    const uint32_t orig = cr.cache;            // A is ranked against the cache before the pass
+    uint32_t left = valid & ~orig;             // non-residents not yet taken
     int pro = 0;
-    {
-        uint32_t kS[V];
-        uint32_t u = 0u;                                       // best key outside the cache
+#pragma unroll 1
+    for (int j = 0; j < R; ++j) {
+        // the best remaining non-resident: largest key, then lowest index
+        uint32_t m[V];
+#pragma unroll
+        for (int v = 0; v < V; ++v) m[v] = ((left >> v) & 1u) ? kS[v] : 0u;
+        uint32_t best = m[0];
+#pragma unroll
+        for (int v = 1; v < V; ++v) best = umax(best, m[v]);
+        const uint32_t mx = __reduce_max_sync(kFull, best);
+        if (mx == 0u) break;                   // no non-resident left
+        const int owner = __ffs(__ballot_sync(kFull, best == mx)) - 1;
+        uint32_t cs = 0u;
+#pragma unroll
+        for (int v = V - 1; v >= 0; --v) cs = m[v] == mx ? (uint32_t)v : cs;   // lowest such slot
+        // residents of the original cache ahead of c: higher keys, and equal
+        // keys at lower indices (lanes before the owner; the owner's slots before c's)
+        uint32_t gt = 0u, eq = 0u;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-            // s^ST = a^T + p^S_rho (a = s^T of the previous token; Spatio-only: p^R)
-            kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;
-            if (!((cr.cache >> v) & 1u)) u = kS[v] > u ? kS[v] : u;
+            const bool res = ((orig >> v) & 1u) != 0u;
+            gt += (res && kS[v] > mx) ? 1u : 0u;
+            eq += (res && kS[v] == mx) ? 1u : 0u;
         }
-        // When at least R experts score strictly above every non-resident one,
-        // the first R candidates are all resident and the pass changes nothing.
-        const uint32_t u1 = __reduce_max_sync(kFull, u);
-        uint32_t above = 0u;
+        const uint32_t tot = __reduce_add_sync(kFull, gt | (eq << 16));
+        uint32_t ahead = tot & 0xffffu;
+        if ((tot >> 16) != 0u) {               // equal keys: count those before c by index
+            const uint32_t c_slot = __shfl_sync(kFull, cs, owner);
+            uint32_t before = 0u;
 #pragma unroll
-        for (int v = 0; v < V; ++v) above += kS[v] > u1 ? 1u : 0u;
-        const bool idle = u1 == 0u || (int)__reduce_add_sync(kFull, above) >= R;
-        KeyList<V> A;
-#pragma unroll
-        for (int v = 0; v < V; ++v) {
-            A.k[v] = kS[v];
-            A.s[v] = v;
+            for (int v = 0; v < V; ++v) {
+                const bool res = ((orig >> v) & 1u) != 0u;
+                before += (res && kS[v] == mx && (lane < owner || (lane == owner && (uint32_t)v < c_slot)))
+                              ? 1u : 0u;
+            }
+            ahead += __reduce_add_sync(kFull, before);
         }
-        if (!idle) presort<V>(A);
-        for (int r = 0; r < (idle ? 0 : R); ++r) {            // candidates, descending
-            uint32_t ke, slot = 0u;
-            const int owner = warp_pop_first<V>(A, lane, ke, slot);
-            if (owner < 0) break;
-            const uint32_t bit = (lane == owner) ? (1u << slot) : 0u;
-            if (__any_sync(kFull, (cr.cache & bit) != 0u)) continue;   // resident
-            if (cr.count < C) {                                // free slot: proactive load
-                cr.cache |= bit;
-                ++cr.count;
-                ++pro;
-                continue;
-            }
-            uint32_t kv, vslot = 0u;
-            const int vo = warp_last_member<V>(kS, cr.cache, lane, kv, vslot);
-            if (ke > kv) {                                     // strictly higher: replace lowest
-                if (lane == vo) cr.cache &= ~(1u << vslot);
-                cr.cache |= bit;
-                ++pro;
-            } else {
-                break;                                         // later candidates lose as well
-            }
+        if (j + (int)ahead >= R) break;        // c is not among the top R, nor is any later one
+        const uint32_t cbit = (lane == owner) ? (1u << cs) : 0u;
+        left &= ~cbit;
+        if (cr.count < C) {                    // free slot: proactive load
+            cr.cache |= cbit;
+            ++cr.count;
+            ++pro;
+            continue;
+        }
+        uint32_t kv, vslot = 0u;
+        const int vo = warp_last_member<V>(kS, cr.cache, lane, kv, vslot);
+        if (mx > kv) {                         // strictly higher: replace the lowest resident
+            const uint32_t vbit = (lane == vo) ? (1u << vslot) : 0u;
+            cr.cache = (cr.cache & ~vbit) | cbit;
+            ++pro;
+        } else {
+            break;                             // later candidates are no higher
         }
     }
     return pro;
 }
 
+// Refinement, access and UpdateCache of one access, given s^T = p^R + p^T,
+// the Spatio prediction of the predecessor and the native Top-K set `sel`
+// (this lane's V bits).  Updates the chain registers; returns the number of
+// proactive loads and writes the demand misses to *n_miss.
 template <int V, bool ALL_VALID>
 __device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V],
                                           const float (&pS)[V], bool refine, uint32_t valid,
@@ -377,10 +406,9 @@ __device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V]
         for (int i = 0; i < nD - freeslots; ++i) {
             uint32_t kv, vslot = 0u;
             const int vo = warp_last_member<V>(kT, vset, lane, kv, vslot);
-            if (lane == vo) {
-                vset &= ~(1u << vslot);
-                cr.cache &= ~(1u << vslot);
-            }
+            const uint32_t rm = (lane == vo) ? (1u << vslot) : 0u;
+            vset &= ~rm;
+            cr.cache &= ~rm;
         }
         cr.count = C;
     } else {
