@@ -502,10 +502,18 @@ __device__ __forceinline__ uint32_t lane_bits(const uint32_t* words, int lane, i
     return (words[e0 >> 5] >> (e0 & 31)) & ((1u << V) - 1u);
 }
 
+// Warps (chains) per block of the stand-alone scans.  The scans are
+// issue-bound with every chain resident at once, so their time is that of the
+// most loaded SM: one-warp blocks spread the B*L chains within one warp per SM
+// of even (3,072 chains over 152 SMs: 20 or 21 warps each, where blocks of
+// four put 24 on some SMs and 20 on the rest).
+constexpr int kScanWarps = 1;
+
 template <int V, bool ALL_VALID, int KP>
-__global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArgs a) {
+__global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWarps)
+    cache_scan_kernel(ScanArgs a) {
     // Top-K sets of the next 32 tokens of each warp's chain, one row per token
-    __shared__ uint32_t sel_s[4][32][8];
+    __shared__ uint32_t sel_s[kScanWarps][32][8];
     StateHeader* hdr = reinterpret_cast<StateHeader*>(a.state);
     const StateLayout lay = state_layout(a.B, a.L, a.N);
     ChainState* chains = reinterpret_cast<ChainState*>(a.state + lay.chains);
@@ -563,7 +571,7 @@ __global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_kernel(ScanArg
         // Without a trace only the Top-K *set* is needed: it does not depend on
         // the cache, so lane j computes it for token t + j ahead of the chain.
         const bool batch_sel = a.trace_topk == nullptr;
-        uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) & 3];
+        uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) % kScanWarps];
         const float* row_base = a.scores + ((size_t)b * T * L + l) * row;   // token 0 of chain
 
         Vec<V> cR = load_vec<V>(unit_ptr(0, l), has && unit_ok(0, l));

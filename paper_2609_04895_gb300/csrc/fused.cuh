@@ -2,7 +2,7 @@
 // scan run in ONE persistent kernel, so the router probabilities never reach
 // HBM (they live in an L2-sized ring of tiles in the workspace).
 //
-// Per CTA (one per SM, cooperative launch so that all CTAs are resident):
+// Per CTA (one per SM, cooperative launch so that all CTAs are resident), 12 warps:
 //   warp 0      TMA producer  (hidden tile + [3N x 64] weight slab per stage)
 //   warp 1      TMEM owner, tcgen05.mma issuer
 //   warps 2..5  epilogue: per tile row (thread = row) the three softmaxes,
@@ -378,7 +378,11 @@ template <int NH, int H, bool PAIR = false>
 struct FusedCfg {
     using RC = RouterCfg<NH, H>;
     static constexpr int GEMM_WARPS = 6;
-    static constexpr int SCAN_WARPS = 10;
+    // six scan warps keep up with the GEMM once the scan step is cheap; more
+    // of them only take issue slots from the epilogue (measured: 6 -> 4.20 ms,
+    // 7 -> 4.24, 8 -> 4.29, 10 -> 4.35 on the Qwen3-30B shape; 5 and 4 fall
+    // behind the tiles, 4.36 and 4.96)
+    static constexpr int SCAN_WARPS = 6;
     static constexpr int THREADS = 32 * (GEMM_WARPS + SCAN_WARPS);
     static constexpr int B_ROWS = PAIR ? RC::NCOL / 2 : RC::NCOL;        // weight rows per CTA
     static constexpr int B_BOX_ROWS = PAIR ? RC::NCH / 2 : RC::B_BOX_ROWS;

@@ -30,7 +30,7 @@ int launch_policy_t(const crc_problem& p, const float* scores, int T, void* stat
     a.policy = policy;
     a.lambda2 = lambda2;
     const int chains = p.B * p.L;
-    const int warps_per_block = 4;
+    const int warps_per_block = kScanWarps;
     const int grid = (chains + warps_per_block - 1) / warps_per_block;
     {
         ProfScope prof(CRC_KERNEL_SCAN, stream);

@@ -135,7 +135,8 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
 }
 
 template <int V, bool ALL_VALID>
-__global__ void __launch_bounds__(128, V >= 8 ? 3 : 6) cache_scan_policy_kernel(PolicyArgs pa) {
+__global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWarps)
+    cache_scan_policy_kernel(PolicyArgs pa) {
     const ScanArgs& a = pa.s;
     StateHeader* hdr = reinterpret_cast<StateHeader*>(a.state);
     const StateLayout lay = state_layout(a.B, a.L, a.N);

@@ -53,7 +53,7 @@ static int launch_scan_t(const crc_problem& p, const float* scores, int T, void*
     a.trace_after = trace ? trace->cache_after_dev : nullptr;
     a.trace_sel = trace ? trace->topk_set_dev : nullptr;
     const int chains = p.B * p.L;
-    const int warps_per_block = 4;
+    const int warps_per_block = kScanWarps;
     const int grid = (chains + warps_per_block - 1) / warps_per_block;
     {
         ProfScope prof(CRC_KERNEL_SCAN, stream);
