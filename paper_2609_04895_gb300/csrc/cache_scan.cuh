@@ -573,6 +573,15 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
         const bool batch_sel = a.trace_topk == nullptr;
         uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) % kScanWarps];
         const float* row_base = a.scores + ((size_t)b * T * L + l) * row;   // token 0 of chain
+        // running pointer to this lane's part of unit (b, t, l); p^S of rho(t, l)
+        // sits at a fixed offset from it: unit (t, l-1), or (t-1, L-1) for l = 0
+        const size_t tok = (size_t)L * row;
+        const ptrdiff_t s_off = l > 0 ? (ptrdiff_t)2 * N - (ptrdiff_t)row
+                                      : (ptrdiff_t)(L - 1) * (ptrdiff_t)row - (ptrdiff_t)tok +
+                                            (ptrdiff_t)2 * N;
+        const float* up = unit_ptr(0, l);
+        const bool traced = a.trace_topk || a.trace_miss || a.trace_pro || a.trace_mid ||
+                            a.trace_after || a.trace_sel;
 
         Vec<V> cR = load_vec<V>(unit_ptr(0, l), has && unit_ok(0, l));
         Vec<V> cT = load_vec<V>(unit_ptr(0, l) + N, has && unit_ok(0, l));
@@ -596,19 +605,33 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
             Vec<V> nR, nT, nS;
             if (t + 1 < T) {
                 const bool ok1 = unit_ok(t + 1, l);
-                nR = load_vec<V>(unit_ptr(t + 1, l), has && ok1);
-                nT = load_vec<V>(unit_ptr(t + 1, l) + N, has && ok1);
-                nS = load_vec<V>(pred_ptr(t + 1), has && want_s &&
-                                                      (l > 0 ? unit_ok(t + 1, l - 1) : unit_ok(t, L - 1)));
+                const float* un = up + tok;
+                nR = load_vec<V>(un, has && ok1);
+                nT = load_vec<V>(un + N, has && ok1);
+                nS = load_vec<V>(un + s_off, has && want_s &&
+                                                 (l > 0 ? unit_ok(t + 1, l - 1) : unit_ok(t, L - 1)));
             }
-            const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
-            scan_step<V, ALL_VALID>(cr, cR.v, cT.v, cS.v, want_s && (t0 + t >= 1), valid, lane, a.K, a.C,
-                         a.R, batch_sel, sel_in, a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
-                         a.trace_miss ? a.trace_miss + unit : nullptr,
-                         a.trace_pro ? a.trace_pro + unit : nullptr,
-                         a.trace_mid ? a.trace_mid + unit * (size_t)((N + 31) >> 5) : nullptr,
-                         a.trace_after ? a.trace_after + unit * (size_t)((N + 31) >> 5) : nullptr,
-                         N, a.trace_sel ? a.trace_sel + unit * (size_t)((N + 31) >> 5) : nullptr);
+            up += tok;
+            const bool refine = want_s && (t0 + t >= 1);
+            if (traced) {
+                const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
+                const size_t NWs = (size_t)((N + 31) >> 5);
+                scan_step<V, ALL_VALID>(cr, cR.v, cT.v, cS.v, refine, valid, lane, a.K, a.C, a.R,
+                                        batch_sel, sel_in,
+                                        a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
+                                        a.trace_miss ? a.trace_miss + unit : nullptr,
+                                        a.trace_pro ? a.trace_pro + unit : nullptr,
+                                        a.trace_mid ? a.trace_mid + unit * NWs : nullptr,
+                                        a.trace_after ? a.trace_after + unit * NWs : nullptr, N,
+                                        a.trace_sel ? a.trace_sel + unit * NWs : nullptr);
+            } else {                      // no trace: the set-valued Top-K, straight to the step
+                float sT[V];
+#pragma unroll
+                for (int v = 0; v < V; ++v) sT[v] = __fadd_rn(cR.v[v], cT.v[v]);
+                int nD;
+                scan_apply<V, ALL_VALID>(cr, sT, cS.v, refine, valid, lane, a.K, a.C, a.R, sel_in,
+                                         &nD);
+            }
             // debug builds: every expert the step made resident lies in this
             // lane's range and the cache holds at most C experts
             (void)CRC_IN_BOUNDS((cr.cache & ~valid) == 0u && cr.count <= a.C, err);
