@@ -5,7 +5,7 @@
 namespace crc {
 namespace {
 
-template <int V, bool ALL_VALID>
+template <int V, bool ALL_VALID, int KP>
 int launch_policy_t(const crc_problem& p, const float* scores, int T, void* state,
                     const crc_trace* trace, int trace_T, int trace_t0, int policy, int lambda2,
                     cudaStream_t stream) {
@@ -34,7 +34,7 @@ int launch_policy_t(const crc_problem& p, const float* scores, int T, void* stat
     const int grid = (chains + warps_per_block - 1) / warps_per_block;
     {
         ProfScope prof(CRC_KERNEL_SCAN, stream);
-        cache_scan_policy_kernel<V, ALL_VALID><<<grid, 32 * warps_per_block, 0, stream>>>(a);
+        cache_scan_policy_kernel<V, ALL_VALID, KP><<<grid, 32 * warps_per_block, 0, stream>>>(a);
     }
     note_launch();
     return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
@@ -46,16 +46,26 @@ int launch_policy_scan(const crc_problem& p, const float* scores, int T, void* s
                        const crc_trace* trace, int trace_T, int trace_t0, int policy,
                        int lambda2, cudaStream_t stream) {
     if (T <= 0) return CRC_OK;
-#define CRC_POLICY_V(VV)                                                                    \
-    return p.N == 32 * VV ? launch_policy_t<VV, true>(p, scores, T, state, trace, trace_T,  \
-                                                      trace_t0, policy, lambda2, stream)    \
-                          : launch_policy_t<VV, false>(p, scores, T, state, trace, trace_T, \
-                                                       trace_t0, policy, lambda2, stream);
+#define CRC_POLICY_KP(VV, KPV)                                                              \
+    return p.N == 32 * VV                                                                   \
+               ? launch_policy_t<VV, true, KPV>(p, scores, T, state, trace, trace_T,        \
+                                                trace_t0, policy, lambda2, stream)          \
+               : launch_policy_t<VV, false, KPV>(p, scores, T, state, trace, trace_T,       \
+                                                 trace_t0, policy, lambda2, stream);
+#define CRC_POLICY_V(VV)                    \
+    {                                       \
+        if (p.K <= 2) CRC_POLICY_KP(VV, 2)  \
+        if (p.K <= 4) CRC_POLICY_KP(VV, 4)  \
+        if (p.K <= 8) CRC_POLICY_KP(VV, 8)  \
+        if (p.K <= 16) CRC_POLICY_KP(VV, 16) \
+        CRC_POLICY_KP(VV, 32)               \
+    }
     if (p.N <= 32) CRC_POLICY_V(1)
     if (p.N <= 64) CRC_POLICY_V(2)
     if (p.N <= 128) CRC_POLICY_V(4)
     CRC_POLICY_V(8)
 #undef CRC_POLICY_V
+#undef CRC_POLICY_KP
 }
 
 }  // namespace crc

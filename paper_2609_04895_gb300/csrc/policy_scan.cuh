@@ -46,7 +46,8 @@ template <int V, bool ALL_VALID>
 __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V],
                                             const float (&pR)[V], const float (&pS)[V],
                                             bool refine, uint32_t valid, int lane,
-                                            const PolicyArgs& a, uint32_t t, uint8_t* topk_out,
+                                            const PolicyArgs& a, uint32_t t, bool have_sel,
+                                            uint32_t sel_in, uint8_t* topk_out,
                                             uint8_t* miss_out, uint8_t* pro_out) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
     const int K = a.s.K, C = a.s.C;
@@ -59,23 +60,27 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
         for (int v = 0; v < V; ++v)
             if ((loaded >> v) & 1u) aux[v] = t;
     }
-    // native Top-K on p^R, in rank order
-    KeyList<V> P;
-#pragma unroll
-    for (int v = 0; v < V; ++v) {
-        P.k[v] = is_valid(v) ? pkey(pR[v]) : 0u;
-        P.s[v] = v;
-    }
-    presort<V>(P);
-    uint32_t sel = 0u;
+    // native Top-K on p^R: given as a set, or popped in rank order when the
+    // trace wants the order
+    uint32_t sel = sel_in;
     int my_topk = 0;
-    for (int k = 0; k < K; ++k) {
-        uint32_t kk, slot = 0u;
-        const int owner = warp_pop_first<V>(P, lane, kk, slot);
-        if (lane == owner) sel |= 1u << slot;
-        if (topk_out) {
-            const int e = __shfl_sync(kFull, lane * V + (int)slot, owner);
-            if (lane == k) my_topk = e;
+    if (!have_sel) {
+        KeyList<V> P;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+            P.k[v] = is_valid(v) ? pkey(pR[v]) : 0u;
+            P.s[v] = v;
+        }
+        presort<V>(P);
+        sel = 0u;
+        for (int k = 0; k < K; ++k) {
+            uint32_t kk, slot = 0u;
+            const int owner = warp_pop_first<V>(P, lane, kk, slot);
+            if (lane == owner) sel |= 1u << slot;
+            if (topk_out) {
+                const int e = __shfl_sync(kFull, lane * V + (int)slot, owner);
+                if (lane == k) my_topk = e;
+            }
         }
     }
     // demand loads; a full cache evicts the lowest priorities outside S (they
@@ -95,10 +100,9 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
         for (int i = 0; i < nD - freeslots; ++i) {
             uint32_t kv, vslot = 0u;
             const int vo = warp_last_member<V>(kV, vset, lane, kv, vslot);
-            if (lane == vo) {
-                vset &= ~(1u << vslot);
-                cr.cache &= ~(1u << vslot);
-            }
+            const uint32_t rm = (lane == vo) ? (1u << vslot) : 0u;
+            vset &= ~rm;
+            cr.cache &= ~rm;
         }
         cr.count = C;
     } else {
@@ -134,9 +138,11 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
     }
 }
 
-template <int V, bool ALL_VALID>
+template <int V, bool ALL_VALID, int KP>
 __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWarps)
     cache_scan_policy_kernel(PolicyArgs pa) {
+    // Top-K sets of the next 32 tokens of each warp's chain, one row per token
+    __shared__ uint32_t sel_s[kScanWarps][32][8];
     const ScanArgs& a = pa.s;
     StateHeader* hdr = reinterpret_cast<StateHeader*>(a.state);
     const StateLayout lay = state_layout(a.B, a.L, a.N);
@@ -191,21 +197,52 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
             return carry_in;
         };
         const bool want_s = pa.policy == CRC_POLICY_SPATIO_LRU && a.R > 0;
+        // without a rank-order trace the Top-K set is taken for 32 tokens at
+        // a time, lane j for token t + j (it does not depend on the cache)
+        const bool batch_sel = a.trace_topk == nullptr;
+        uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) % kScanWarps];
+        const float* row_base = a.scores + ((size_t)b * T * L + l) * row;   // token 0 of chain
+        // running pointer to unit (b, t, l); p^S of rho(t, l) at a fixed offset
+        const size_t tok = (size_t)L * row;
+        const ptrdiff_t s_off = l > 0 ? (ptrdiff_t)2 * N - (ptrdiff_t)row
+                                      : (ptrdiff_t)(L - 1) * (ptrdiff_t)row - (ptrdiff_t)tok +
+                                            (ptrdiff_t)2 * N;
+        const float* up = unit_ptr(0, l);
+        const bool traced = a.trace_topk || a.trace_miss || a.trace_pro;
 
-        Vec<V> cR = load_vec<V>(unit_ptr(0, l), has);
+        Vec<V> cR = load_vec<V>(up, has);
         Vec<V> cS = load_vec<V>(pred_ptr(0), has && want_s && t0 >= 1);
         for (int t = 0; t < T; ++t) {
+            if (batch_sel && (t & 31) == 0) {
+                __syncwarp();
+                if (t + lane < T)
+                    row_topk_mask<KP>(row_base + (size_t)(t + lane) * tok, N, a.K, sel_rows[lane]);
+                __syncwarp();
+            }
+            uint32_t sel_in = 0u;
+            if (batch_sel && has) {
+                const uint32_t e0 = (uint32_t)lane * V;
+                sel_in = (sel_rows[t & 31][e0 >> 5] >> (e0 & 31)) & ((1u << V) - 1u);
+            }
             Vec<V> nR, nS;
             if (t + 1 < T) {
-                nR = load_vec<V>(unit_ptr(t + 1, l), has);
-                nS = load_vec<V>(pred_ptr(t + 1), has && want_s);
+                nR = load_vec<V>(up + tok, has);
+                nS = load_vec<V>(up + tok + s_off, has && want_s);
             }
-            const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
-            policy_step<V, ALL_VALID>(cr, aux, cR.v, cS.v, want_s && (t0 + t >= 1), valid, lane, pa,
-                                      (uint32_t)(t0 + t),
-                                      a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
-                                      a.trace_miss ? a.trace_miss + unit : nullptr,
-                                      a.trace_pro ? a.trace_pro + unit : nullptr);
+            up += tok;
+            const bool refine = want_s && (t0 + t >= 1);
+            if (traced) {
+                const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
+                policy_step<V, ALL_VALID>(cr, aux, cR.v, cS.v, refine, valid, lane, pa,
+                                          (uint32_t)(t0 + t), batch_sel, sel_in,
+                                          a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
+                                          a.trace_miss ? a.trace_miss + unit : nullptr,
+                                          a.trace_pro ? a.trace_pro + unit : nullptr);
+            } else {
+                policy_step<V, ALL_VALID>(cr, aux, cR.v, cS.v, refine, valid, lane, pa,
+                                          (uint32_t)(t0 + t), true, sel_in, nullptr, nullptr,
+                                          nullptr);
+            }
             cR = nR;
             cS = nS;
         }

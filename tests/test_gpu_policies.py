@@ -83,6 +83,23 @@ def test_policy_scan_bit_exact(C, oracle_lib, name, w, quant, policy):
     r, tr = run_gpu(C, w, p32, policy, 1)
     o = oracle_lib.policy_scan(p32, w.K, w.C, w.R, policy, lambda2=1)
     check(r, tr, o, policy)
+    # Without the rank-order Top-K the kernel takes the Top-K set for 32
+    # tokens at a time; untraced, and with misses and proactive loads only,
+    # the results are the same.
+    p = C.problem_of(w)
+    sc = torch.from_numpy(p32).cuda()
+    for traced in (False, True):
+        st = C.State(p)
+        tr2 = C.Trace.alloc(p, w.T, rank_order=False) if traced else None
+        C.cache_scan_policy(p, sc, st, policy, tr2, lambda_halves=1)
+        r2 = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
+        assert r2["error"] == 0
+        for k in ("cache_bits", "chain_counters"):
+            assert np.array_equal(r2[k], r[k]), (traced, k)
+        assert np.array_equal(r2["retention"].view(np.uint32), r["retention"].view(np.uint32))
+        assert np.array_equal(st.read_aux(), r["aux"])
+        if traced:
+            assert torch.equal(tr2.misses, tr.misses) and torch.equal(tr2.proactive, tr.proactive)
 
 
 @pytest.mark.parametrize("lam", [0, 2])
