@@ -11,7 +11,9 @@ writes the whole workload with that re-draw table, the benchmark's fused
 kernel runs over it, and on the sampled streams every per-access decision --
 the native Top-K set (Sec. 2), the demand misses and the proactive loads of
 Algorithm 2, the final caches after Algorithm 1 and the counters -- must
-equal the fp64 oracle's, over all T tokens of every layer.
+equal the fp64 oracle's, over all T tokens of every layer.  Cases: Tiny (all
+four streams), the Qwen3-30B and GPT-OSS-20B shapes (eight streams each) and
+the update-only sweep at C = 16 and C = 96 (four of its 256 streams each).
 """
 import numpy as np
 import pytest
@@ -47,12 +49,16 @@ def _sets(topk: np.ndarray, N: int) -> np.ndarray:
 
 
 CASES = [
+    (S.TINY, (0, 1, 2, 3)),                                          # every stream
     (S.QWEN3_30B, (0, 9, 18, 27, 36, 45, 54, 63)),
     (S.GPT_OSS_20B, (0, 17, 34, 51, 68, 85, 102, 127)),
+    # the update-only sweep (R = 0) at its smallest and largest capacity
+    (S.SWEEP_R0.with_(C=16), (0, 85, 170, 255)),
+    (S.SWEEP_R0.with_(C=96), (0, 85, 170, 255)),
 ]
 
 
-@pytest.mark.parametrize("w,streams", CASES, ids=[c[0].name for c in CASES])
+@pytest.mark.parametrize("w,streams", CASES, ids=[f"{c[0].name}-C{c[0].C}" for c in CASES])
 def test_certified_streams_equal_fp64_oracle(C, oracle_lib, w, streams):
     from oracle import certify
     W = S.weights(w, seed=0)
