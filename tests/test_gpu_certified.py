@@ -130,3 +130,69 @@ def test_certified_streams_equal_fp64_oracle(C, oracle_lib, w, streams):
         traffic = (int(cc[..., 1].sum()) + int(cc[..., 2].sum())) * w.expert_bytes
         oc = cert["counters"]
         assert traffic == (int(oc[..., 1].sum()) + int(oc[..., 2].sum())) * w.expert_bytes
+
+
+@pytest.mark.parametrize("R", S.LARGE.extra["R_values"])
+def test_large_certified_prefix(C, oracle_lib, R):
+    """The large shape (L = 94, d = 4096, B = 512) streamed in 128-token
+    chunks as the benchmark runs it: the first 256 tokens of two sampled
+    streams are drawn margin-certified (a whole stream is a quarter of an hour
+    of fp64 oracle work), the device generator writes both chunks with that
+    re-draw table, and the fused kernel's per-access decisions and the chain
+    states after 256 tokens equal the fp64 oracle's."""
+    from oracle import certify
+    TC, CH = 256, 128
+    w = S.LARGE.with_(R=R)
+    wc = w.with_(T=TC)
+    streams = ((R * 97) % w.B, (R * 97 + 256) % w.B)
+    Wd = C.synth_weights(w.L, w.N, w.d, seed=0)
+    Wb = Wd.view(torch.int16).cpu().numpy().view(np.uint16)
+    cert = certify.certified_streams(wc, Wb, seed=0, streams=streams, tol=TOL)
+    print(f"\nlarge R={R}: {len(streams)} streams x {TC} tokens x {w.L} layers, "
+          f"{int(cert['redraws'].sum())} redraws, certified {float(cert['certified'].mean()):.5f}")
+    assert cert["certified"].mean() >= 0.999
+    p = C.problem_of(w)
+    hbuf = torch.empty((w.B, CH, w.L, w.d), dtype=torch.bfloat16, device="cuda")
+    carry = torch.zeros((w.B, w.L, w.d), dtype=torch.float32, device="cuda")
+    ws = torch.empty(C.crc_fused_workspace_bytes(p), dtype=torch.uint8, device="cuda")
+    st = C.State(p)
+    idx = list(streams)
+    g_set, g_mis, g_pro = [], [], []
+    try:
+        for c in range(TC // CH):
+            t0 = c * CH
+            att = np.zeros((w.B, CH, w.L), np.uint8)
+            att[idx] = cert["attempts"][:, t0:t0 + CH]
+            C.synth_hidden(w.B, CH, w.L, w.d, seed=0, rho_t=w.rho_t, rho_l=w.rho_l, t0=t0,
+                           carry=carry, attempts=torch.from_numpy(att).cuda(), out=hbuf)
+            for i, b in enumerate(idx):
+                ref = torch.from_numpy(cert["hidden"][i, t0:t0 + CH].view(np.int16)).cuda()
+                assert torch.equal(hbuf[b].view(torch.int16), ref), (b, c)
+            tr = C.Trace.alloc(p, CH, rank_order=False, topk_set=True)
+            C.crc_profile_begin()
+            C.route_and_cache(p, hbuf, Wd, st, tr, workspace=ws)
+            assert C.crc_profile_end()["fused"]["launches"] == 1
+            g_set.append(tr.topk_set[idx].cpu().numpy().view(np.uint32))
+            g_mis.append(tr.misses[idx].cpu().numpy())
+            g_pro.append(tr.proactive[idx].cpu().numpy())
+            del tr
+    finally:
+        del hbuf, ws, carry
+        torch.cuda.empty_cache()
+    r = st.read(want_caches=True, want_retention=True, want_chain_counters=True)
+    assert r["error"] == 0 and r["tokens"] == TC
+    g_set, g_mis, g_pro = (np.concatenate(x, axis=1) for x in (g_set, g_mis, g_pro))
+    o_set = _sets(cert["topk"], w.N)
+    for i, b in enumerate(idx):
+        for l in range(w.L):
+            bad = np.flatnonzero(~cert["certified"][i, :, l])
+            stop = int(bad[0]) if len(bad) else TC
+            sl = slice(0, stop)
+            assert np.array_equal(g_set[i, sl, l], o_set[i, sl, l]), (b, l)
+            assert np.array_equal(g_mis[i, sl, l], cert["misses"][i, sl, l]), (b, l)
+            assert np.array_equal(g_pro[i, sl, l], cert["proactive"][i, sl, l]), (b, l)
+            if stop == TC:
+                assert np.array_equal(r["cache_bits"][b, l], cert["cache_bits"][i, l])
+                assert np.array_equal(r["chain_counters"][b, l], cert["counters"][i, l])
+                ref = cert["aT"][i, l]
+                assert (np.abs(r["retention"][b, l].astype(np.float64) - ref) / ref).max() <= TOL
