@@ -1,8 +1,12 @@
 // Fused route-and-cache: the router heads on the tensor cores and the cache
-// scan run in ONE persistent kernel, so the router probabilities never reach
-// HBM (they live in an L2-sized ring of tiles in the workspace).
+// scan run in ONE persistent kernel: the router probabilities are never
+// written out as scores; each tile's record (Top-K set, s^T, p^S: 1.04 KB per
+// decision for N = 128) passes through a ring of three token blocks of tiles
+// in the workspace, read once by the scan warps (from L2 when the scan keeps
+// up, else written back to DRAM and read from there).
 //
-// Per CTA (one per SM, cooperative launch so that all CTAs are resident), 12 warps:
+// Per CTA (one per SM, cooperative launch so that all CTAs are resident), 12 warps
+// (14 when R > 4):
 //   warp 0      TMA producer  (hidden tile + [3N x 64] weight slab per stage)
 //   warp 1      TMEM owner, tcgen05.mma issuer
 //   warps 2..5  epilogue: per tile row (thread = row) the three softmaxes,
@@ -378,12 +382,21 @@ template <int NH, int H, bool PAIR = false>
 struct FusedCfg {
     using RC = RouterCfg<NH, H>;
     static constexpr int GEMM_WARPS = 6;
-    // six scan warps keep up with the GEMM once the scan step is cheap; more
-    // of them only take issue slots from the epilogue (measured: 6 -> 4.20 ms,
-    // 7 -> 4.24, 8 -> 4.29, 10 -> 4.35 on the Qwen3-30B shape; 5 and 4 fall
-    // behind the tiles, 4.36 and 4.96)
+    // Scan warps per CTA, chosen at launch from the refinement budget.  Six
+    // keep up with the GEMM when R <= 4; more of them only take issue slots
+    // from the epilogue (Qwen3-30B shape: 6 -> 4.20 ms, 7 -> 4.24, 8 -> 4.29,
+    // 10 -> 4.35; 5 and 4 fall behind the tiles, 4.36 and 4.96).  With R = 8
+    // a step has up to twice the refinement rounds and six fall behind (one
+    // 128-token chunk of the Qwen3-235B shape: 15.9 ms with 6, 15.25 with 8,
+    // 15.17 with 10; with R = 2: 14.7-15.0 with 6 or 8).  The kernel's roles
+    // do not depend on the count: every warp past the GEMM warps scans.
     static constexpr int SCAN_WARPS = 6;
+    static constexpr int SCAN_WARPS_WIDE = 8;
     static constexpr int THREADS = 32 * (GEMM_WARPS + SCAN_WARPS);
+    static constexpr int MAX_THREADS = 32 * (GEMM_WARPS + SCAN_WARPS_WIDE);
+    static int threads_for(int R) {
+        return 32 * (GEMM_WARPS + (R > 4 ? SCAN_WARPS_WIDE : SCAN_WARPS));
+    }
     static constexpr int B_ROWS = PAIR ? RC::NCOL / 2 : RC::NCOL;        // weight rows per CTA
     static constexpr int B_BOX_ROWS = PAIR ? RC::NCH / 2 : RC::B_BOX_ROWS;
     static constexpr int B_BOXES = B_ROWS / B_BOX_ROWS;

@@ -81,7 +81,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
             at[0].val.clusterDim.z = 1;
             cudaLaunchConfig_t c = {};
             c.gridDim = dim3((unsigned)(sm_count() / 2 * 2));
-            c.blockDim = dim3(Cfg::THREADS);
+            c.blockDim = dim3(Cfg::MAX_THREADS);
             c.dynamicSmemBytes = Cfg::SMEM_BYTES;
             c.attrs = at;
             c.numAttrs = 1;
@@ -95,7 +95,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
             grid = std::min(2 * ncl, sm_count() / 2 * 2);
         } else {
             int per_sm = 0;
-            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Cfg::THREADS,
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Cfg::MAX_THREADS,
                                                               Cfg::SMEM_BYTES) != cudaSuccess ||
                 per_sm < 1) {
                 (void)cudaGetLastError();
@@ -140,6 +140,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
     a.tr_after = trace ? trace->cache_after_dev : nullptr;
     a.tr_sel = trace ? trace->topk_set_dev : nullptr;
     void* args[] = {(void*)&mh, (void*)&mw, (void*)&a};
+    const int threads = Cfg::threads_for(p.R);
     cudaError_t e;
     if (PAIR) {
         cudaLaunchAttribute at[2];
@@ -151,7 +152,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
         at[1].val.cooperative = 1;
         cudaLaunchConfig_t c = {};
         c.gridDim = dim3((unsigned)grid);
-        c.blockDim = dim3(Cfg::THREADS);
+        c.blockDim = dim3(threads);
         c.dynamicSmemBytes = Cfg::SMEM_BYTES;
         c.stream = stream;
         c.attrs = at;
@@ -172,7 +173,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
         }
     } else {
         ProfScope prof(CRC_KERNEL_FUSED, stream);
-        e = cudaLaunchCooperativeKernel((const void*)kern, grid, Cfg::THREADS, args,
+        e = cudaLaunchCooperativeKernel((const void*)kern, grid, threads, args,
                                         Cfg::SMEM_BYTES, stream);
     }
     note_launch();
