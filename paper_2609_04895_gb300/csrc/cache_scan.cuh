@@ -159,7 +159,7 @@ struct ChainRegs {
 
 // ---------------------------------------------------------------------------
 // Thread-serial Top-K set of one score row (used for many tokens at once, one
-// token per lane).  A bitonic network on fp32 values (max/min only) finds the
+// token per lane).  Sorting networks on fp32 values (max/min only) find the
 // K-th largest value theta; a second pass in index order takes every value
 // above theta and, among values equal to theta, the lowest indices -- exactly
 // the first K under (score desc, index asc).
@@ -170,7 +170,8 @@ constexpr int pow2_at_least(int x) {
     return p;
 }
 
-// Sort P values descending (P a power of two), fully unrolled.
+// Sort P values descending (P a power of two), fully unrolled: the bitonic
+// network.
 template <int P>
 __device__ __forceinline__ void bitonic_sort_desc(float (&a)[P]) {
 #pragma unroll
@@ -188,6 +189,37 @@ __device__ __forceinline__ void bitonic_sort_desc(float (&a)[P]) {
                     } else {
                         a[i] = lo;
                         a[l] = hi;
+                    }
+                }
+            }
+        }
+    }
+}
+
+// The same with Batcher's odd-even merge sort, which sorts P = 4 with 5
+// compare-exchanges and P = 8 with 19 (the bitonic network takes 6 and 24).
+// Stage p merges sorted runs of p into runs of 2p; within it, the
+// compare-exchanges at distance k join elements of the same run of 2p.  Used
+// up to P = 8; beyond that the compiler no longer resolves every index.
+template <int P>
+__device__ __forceinline__ void sort_desc(float (&a)[P]) {
+    if constexpr (P > 8) {
+        bitonic_sort_desc<P>(a);
+    } else {
+#pragma unroll
+        for (int p = 1; p < P; p <<= 1) {
+#pragma unroll
+            for (int k = p; k >= 1; k >>= 1) {
+#pragma unroll
+                for (int j = k % p; j + k < P; j += 2 * k) {
+#pragma unroll
+                    for (int i = 0; i < k; ++i) {
+                        const int x = i + j, y = i + j + k;
+                        if (y < P && x / (2 * p) == y / (2 * p)) {
+                            const float hi = fmaxf(a[x], a[y]), lo = fminf(a[x], a[y]);
+                            a[x] = hi;
+                            a[y] = lo;
+                        }
                     }
                 }
             }
@@ -231,7 +263,7 @@ struct TopKAcc {
             float b[KP];
 #pragma unroll
             for (int i = 0; i < KP; ++i) b[i] = (i < G) ? x[g + i] : -1.0f;
-            bitonic_sort_desc<KP>(b);
+            sort_desc<KP>(b);
             merge_top_desc<KP>(run, b);
         }
     }
@@ -285,6 +317,23 @@ __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, ui
         acc.add16(x);
     }
     const float th = acc.theta(K);
+    // Every score >= theta: the Top-K set exactly when no more scores equal
+    // theta than the set takes (the usual case), i.e. when it has K members.
+    int cnt = 0;
+    for (int c = 0; c < N; c += 32) {
+        uint32_t w = 0u;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            if (c + 4 * q >= N) break;
+            const float4 f = __ldg(reinterpret_cast<const float4*>(row + c) + q);
+            w |= ((f.x >= th ? 1u : 0u) | (f.y >= th ? 2u : 0u) | (f.z >= th ? 4u : 0u) |
+                  (f.w >= th ? 8u : 0u)) << (4 * q);
+        }
+        mask[c >> 5] = w;
+        cnt += __popc(w);
+    }
+    if (cnt == K) return;
+    // surplus scores equal to theta: take the lowest indices among them
     int need = acc.need(K, th);
     for (int c = 0; c < N; c += 32) {
         uint32_t w = 0u;
@@ -305,14 +354,13 @@ __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, ui
 //
 // Only the non-resident members of A can change the cache, so they are taken
 // one at a time in order -- the best remaining non-resident c -- and c is a
-// member of A exactly when fewer than R experts precede it in the order: the j
-// non-residents already loaded and the residents of the original cache ahead
-// of it.  The first such count is also the test that leaves the cache alone
-// when at least R residents precede every non-resident.  An original resident
-// that a candidate evicted is never taken as a candidate itself: in the
-// literal loop it would meet a cache whose lowest member is no lower than it
-// and lose the strict test, ending the pass exactly as the rank test or the
-// strict test ends it here.
+// member of A = Top_R exactly when fewer than R experts precede it in the
+// order (its rank).  The first rank test is also the one that leaves the cache
+// alone when the R first experts are all resident.  An original resident that
+// a candidate evicted is never taken as a candidate itself: in the literal
+// loop it would meet a cache whose lowest member is no lower than it and lose
+// the strict test, ending the pass exactly as the rank test or the strict
+// test ends it here.
 template <int V, bool ALL_VALID>
 __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V], uint32_t valid,
                                            int lane, int C, int R) {
@@ -321,8 +369,7 @@ __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V
 #pragma unroll
     for (int v = 0; v < V; ++v)
         kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;
-    const uint32_t orig = cr.cache;            // A is ranked against the cache before the pass
-    uint32_t left = valid & ~orig;             // non-residents not yet taken
+    uint32_t left = valid & ~cr.cache;         // non-residents not yet taken
     int pro = 0;
 #pragma unroll 1
     for (int j = 0; j < R; ++j) {
@@ -339,29 +386,27 @@ __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V
         uint32_t cs = 0u;
 #pragma unroll
         for (int v = V - 1; v >= 0; --v) cs = m[v] == mx ? (uint32_t)v : cs;   // lowest such slot
-        // residents of the original cache ahead of c: higher keys, and equal
-        // keys at lower indices (lanes before the owner; the owner's slots before c's)
+        // rank of c: experts with higher keys, and with equal keys at lower
+        // indices (lanes before the owner; the owner's slots before c's).
+        // Invalid slots hold key 0 and count for neither.
         uint32_t gt = 0u, eq = 0u;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-            const bool res = ((orig >> v) & 1u) != 0u;
-            gt += (res && kS[v] > mx) ? 1u : 0u;
-            eq += (res && kS[v] == mx) ? 1u : 0u;
+            gt += kS[v] > mx ? 1u : 0u;
+            eq += kS[v] == mx ? 1u : 0u;
         }
         const uint32_t tot = __reduce_add_sync(kFull, gt | (eq << 16));
-        uint32_t ahead = tot & 0xffffu;
-        if ((tot >> 16) != 0u) {               // equal keys: count those before c by index
+        uint32_t rank = tot & 0xffffu;
+        if ((tot >> 16) > 1u) {                // c shares its key: count those before it by index
             const uint32_t c_slot = __shfl_sync(kFull, cs, owner);
             uint32_t before = 0u;
 #pragma unroll
-            for (int v = 0; v < V; ++v) {
-                const bool res = ((orig >> v) & 1u) != 0u;
-                before += (res && kS[v] == mx && (lane < owner || (lane == owner && (uint32_t)v < c_slot)))
+            for (int v = 0; v < V; ++v)
+                before += (kS[v] == mx && (lane < owner || (lane == owner && (uint32_t)v < c_slot)))
                               ? 1u : 0u;
-            }
-            ahead += __reduce_add_sync(kFull, before);
+            rank += __reduce_add_sync(kFull, before);
         }
-        if (j + (int)ahead >= R) break;        // c is not among the top R, nor is any later one
+        if ((int)rank >= R) break;             // c is not among the top R, nor is any later one
         const uint32_t cbit = (lane == owner) ? (1u << cs) : 0u;
         left &= ~cbit;
         if (cr.count < C) {                    // free slot: proactive load

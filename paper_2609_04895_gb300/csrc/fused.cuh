@@ -10,8 +10,8 @@
 //   warp 0      TMA producer  (hidden tile + [3N x 64] weight slab per stage)
 //   warp 1      TMEM owner, tcgen05.mma issuer
 //   warps 2..5  epilogue: per tile row (thread = row) the three softmaxes,
-//               s^T = p^R + p^T, the Top-K set of p^R (bitonic network on the
-//               values, then an exact threshold-and-ties pass) and p^S; the
+//               s^T = p^R + p^T, the Top-K set of p^R (sorting networks on
+//               the values, then an exact threshold-and-ties pass) and p^S; the
 //               row's record (Top-K mask, s^T, p^S) goes to a ring slot with
 //               coalesced stores, then the tile is published
 //   warps 6..   scan warps: take items (chain, block of TB tokens) in token
