@@ -232,7 +232,7 @@ KERNEL_SOURCES = {
     "router": ["router.cu", "router_gemm.cuh", "crc_device.cuh"],
     "scan": ["scan.cu", "cache_scan.cuh", "crc_device.cuh"],
     "policy": ["policy.cu", "policy_scan.cuh", "cache_scan.cuh", "crc_device.cuh"],
-    "loss": ["loss.cu"],
+    "loss": ["loss.cu", "cache_scan.cuh", "crc_device.cuh"],
 }
 
 
@@ -448,8 +448,12 @@ def run_loss(args, P, C, w, p, dev, stream, rank, world):
     per_unit = 24.0 * w.N + 8.0
     avg_ms = kt["loss"]["ms"] / max(1, kt["loss"]["launches"])
     achieved = per_unit * w.units / (avg_ms / 1000.0) / 1e9
-    V = 1 if w.N <= 32 else 2 if w.N <= 64 else 4 if w.N <= 128 else 8
-    kname = f"cache_loss_kernel<{V}>"
+    if w.N in (16, 32) and top_b <= 16:         # short rows: 16 elements per lane
+        kp = 2 if top_b <= 2 else 4 if top_b <= 4 else 8 if top_b <= 8 else 16
+        kname = f"cache_loss_rows_kernel<{w.N // 16},{kp}>"
+    else:
+        V = 1 if w.N <= 32 else 2 if w.N <= 64 else 4 if w.N <= 128 else 8
+        kname = f"cache_loss_kernel<{V}>"
     tr, _ = committed_traffic(kname, w.name)
     roof = {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
             "frac": achieved / pk["hbm_gbs"], "traffic": None if tr is None else tr * w.units,

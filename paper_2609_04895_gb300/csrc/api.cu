@@ -452,8 +452,7 @@ int crc_host_free(void* ptr) {
 
 size_t crc_loss_workspace_bytes(const crc_problem* p, int32_t T) {
     if (check_problem(p, false) != CRC_OK || T < 1) return 0;
-    const LossPlan pl = loss_plan(p->B, p->L, T);
-    const size_t bytes = (size_t)p->B * p->L * pl.nchunks * 2 * sizeof(double);
+    const size_t bytes = (size_t)loss_task_slots(p->B, p->L, T, p->N) * 2 * sizeof(double);
     return (bytes + 255) / 256 * 256;
 }
 

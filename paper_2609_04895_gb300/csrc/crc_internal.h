@@ -73,6 +73,10 @@ struct LossPlan {
     int nchunks, chunk;
 };
 LossPlan loss_plan(int B, int L, int T);
+// Per-task partial sums the loss kernels may write (the workspace of
+// crc_cache_loss): the plan's tasks, or for N <= 32, whose chunks are sized
+// at launch, B * L tasks per 32 tokens.
+long long loss_task_slots(int B, int L, int T, int N);
 int launch_cache_loss(const crc_problem& p, const float* probs, int T, int heads, int top_b,
                       double tau, double w_T, double w_ST, float* loss, double* means,
                       float* grad, void* workspace, cudaStream_t stream);

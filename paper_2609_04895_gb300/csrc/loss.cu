@@ -34,12 +34,14 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
+#include "cache_scan.cuh"
 #include "crc_internal.h"
 
 namespace crc {
 namespace {
 
-constexpr unsigned kFull = 0xffffffffu;
 constexpr int kLossWarps = 8;
 
 struct LossArgs {
@@ -473,6 +475,416 @@ __global__ void __launch_bounds__(32 * kLossWarps, loss_blocks<V>()) cache_loss_
     }
 }
 
+// ---------------------------------------------------------------------------
+// Short rows (N = 16 or 32, top_b <= 16).  One warp-wide reduction per row
+// quantity leaves such rows latency- and issue-bound, so here a row is held
+// by NL = N / 16 lanes, 16 elements each, a warp runs 32 / NL tasks side by
+// side, and every per-row quantity is lane-serial work plus at most one
+// exchange with the partner lane (shuffle xor 1).  theta_B is the top_b-th
+// entry of the running top KP (sorting networks over the lane's 16 values,
+// merged with the partner's), e* the need-th value equal to it in index
+// order; per element the arithmetic is that of the warp-per-row kernel.
+// ---------------------------------------------------------------------------
+constexpr int kRowE = 16;       // row elements per lane
+constexpr int kRowWarps = 4;    // warps per block of the short-row kernel
+
+template <int NL>
+__device__ __forceinline__ float pair_sum(float x) {
+    if constexpr (NL == 2) x += __shfl_xor_sync(kFull, x, 1);
+    return x;
+}
+
+__device__ __forceinline__ void load16(float (&x)[kRowE], const float* p, bool ok) {
+    if (!ok) {
+#pragma unroll
+        for (int j = 0; j < kRowE; ++j) x[j] = 0.f;
+        return;
+    }
+#pragma unroll
+    for (int i = 0; i < kRowE / 4; ++i) {
+        const float4 v = __ldcs(reinterpret_cast<const float4*>(p) + i);
+        x[4 * i] = v.x;
+        x[4 * i + 1] = v.y;
+        x[4 * i + 2] = v.z;
+        x[4 * i + 3] = v.w;
+    }
+}
+
+__device__ __forceinline__ void store16(float* p, const float (&x)[kRowE]) {
+#pragma unroll
+    for (int i = 0; i < kRowE / 4; ++i)
+        __stcs(reinterpret_cast<float4*>(p) + i,
+               make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]));
+}
+
+// 16-byte asynchronous copy global -> shared (zero-filled when !ok; the
+// address is then not read), and its group fences.
+__device__ __forceinline__ void cp_async16(float4* smem, const float* gmem, bool ok) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(smem)),
+                 "l"(gmem), "r"(ok ? 16 : 0)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait1() {
+    asm volatile("cp.async.wait_group 1;" ::: "memory");
+}
+
+// theta_B of the row (the same in both lanes of a pair) and, in `slot`, this
+// lane's slot holding e*, the element at position top_b of the order (score
+// descending, index ascending), or -1.  The lower lane of a pair holds
+// elements 0-15, the upper 16-31.
+template <int NL, int KP>
+__device__ __forceinline__ float row_theta(const float (&s)[kRowE], int top_b, int half, int lane,
+                                           int& slot) {
+    // the lane's top KP, descending: sort the groups of KP values, merge them
+    float run[KP];
+#pragma unroll
+    for (int i = 0; i < KP; ++i) run[i] = s[i];
+    sort_desc<KP>(run);
+#pragma unroll
+    for (int g = KP; g < kRowE; g += KP) {
+        float b[KP];
+#pragma unroll
+        for (int i = 0; i < KP; ++i) b[i] = s[g + i];
+        sort_desc<KP>(b);
+        merge_top_desc<KP>(run, b);
+    }
+    if constexpr (NL == 2) {                    // and the partner lane's
+        float o[KP];
+#pragma unroll
+        for (int i = 0; i < KP; ++i) o[i] = __shfl_xor_sync(kFull, run[i], 1);
+        merge_top_desc<KP>(run, o);
+    }
+    float th = run[0];
+#pragma unroll
+    for (int i = 1; i < KP; ++i) th = i == top_b - 1 ? run[i] : th;
+    int above = 0;                              // entries above theta, all within the top KP
+#pragma unroll
+    for (int i = 0; i < KP; ++i) above += (i < top_b && run[i] > th) ? 1 : 0;
+    // e* is the (top_b - above)-th entry equal to theta in index order
+    uint32_t eq = 0u;
+#pragma unroll
+    for (int j = 0; j < kRowE; ++j) eq |= s[j] == th ? 1u << j : 0u;
+    int r = top_b - above;
+    if constexpr (NL == 2) {
+        const int eq_lo = __popc(__shfl_sync(kFull, eq, lane & ~1));
+        if (half) r -= eq_lo;
+    }
+    slot = (r >= 1 && r <= __popc(eq)) ? (int)__fns(eq, 0u, r) : -1;
+    return th;
+}
+
+// Rows of one step in shared memory: float4 i of thread x at st[i][x];
+// quads 0-3 p^T_t, 4-7 p^R_{t+1}, 8-11 p^S_{rho(t+1)} (16 elements each).
+using RowStage = float4[12][32 * kRowWarps];
+
+// One 16-byte shared-memory load, issued where it is written: kept whole
+// (a warp's loads of a quad are then contiguous) and ordered after the
+// cp.async wait.
+__device__ __forceinline__ float4 lds4(const float4& p) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(smem_u32(&p)));
+    return v;
+}
+
+__device__ __forceinline__ float f4(const float4& v, int c) {
+    return c == 0 ? v.x : c == 1 ? v.y : c == 2 ? v.z : v.w;
+}
+
+// One step's two terms from p^R_t (registers), p^T_t, p^S_{rho(t+1)} and the
+// target q = p^R_{t+1} (the stage): returns (l^T, l^ST); dT = dl/dp^T,
+// dR = carry + dT (carry: the target part of p^R_t from the step before),
+// dS = dl/dp^S, all scaled by the objective's coefficients; carry becomes the
+// target part of p^R_{t+1}.  s^T and s^ST are re-formed where they are used,
+// by the same fp32 additions, so they need no registers across the step.
+template <int NL, int KP>
+__device__ __forceinline__ float2 rows_step(const float (&pR)[kRowE], const RowStage& sg, int x,
+                                            bool st, int top_b, const LossArgs& a, int half,
+                                            int lane, float (&carry)[kRowE], float (&dR)[kRowE],
+                                            float (&dT)[kRowE], float (&dS)[kRowE]) {
+    int jT, jST = -1;
+    float thT, thST = 0.f;
+    {
+        float s[kRowE];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float4 f = lds4(sg[i][x]);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) s[4 * i + c] = __fadd_rn(pR[4 * i + c], f4(f, c));
+        }
+        thT = row_theta<NL, KP>(s, top_b, half, lane, jT);
+        if (st) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float4 f = lds4(sg[8 + i][x]);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) s[4 * i + c] = __fadd_rn(s[4 * i + c], f4(f, c));
+            }
+            thST = row_theta<NL, KP>(s, top_b, half, lane, jST);
+        }
+    }
+    const float k2 = a.k2;
+    float lT = 0.f, WT = 0.f, lST = 0.f, WST = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float4 fT = lds4(sg[i][x]), fq = lds4(sg[4 + i][x]);
+        const float4 fS = st ? lds4(sg[8 + i][x]) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int j = 4 * i + c;
+            const float q = f4(fq, c);
+            const float sT = __fadd_rn(pR[j], f4(fT, c));
+            // with d = s - theta, u = sigmoid(|d| / tau), v = 1 - u: 1 - m = v if
+            // d >= 0 else u, and w = q m (1 - m) = q u v
+            const float d = sT - thT;
+            const float E = ex2_approx(-fabsf(d) * k2);
+            const float u = rcp_approx(1.f + E);
+            const float v = E * u;
+            const float om = d >= 0.f ? v : u;
+            lT = fmaf(q, om, lT);
+            const float w = q * (u * v);
+            WT += w;
+            float omS = 0.f, wS = 0.f;
+            if (st) {
+                const float d2 = __fadd_rn(sT, f4(fS, c)) - thST;
+                const float E2 = ex2_approx(-fabsf(d2) * k2);
+                const float u2 = rcp_approx(1.f + E2);
+                const float v2 = E2 * u2;
+                omS = d2 >= 0.f ? v2 : u2;
+                lST = fmaf(q, omS, lST);
+                wS = q * (u2 * v2);
+                WST += wS;
+            }
+            const float gs = -fmaf(a.gT, w, a.gST * wS);
+            dT[j] = gs;
+            dR[j] = carry[j] + gs;
+            dS[j] = -a.gST * wS;
+            carry[j] = fmaf(a.cT, om, a.cST * omS);
+        }
+    }
+    lT = pair_sum<NL>(lT);
+    WT = pair_sum<NL>(WT);
+    lST = pair_sum<NL>(lST);
+    WST = pair_sum<NL>(WST);
+    // through theta_B = s_{e*}: dl/ds_{e*} gains W / tau
+    const float cw = a.gT * WT, cws = a.gST * WST;
+#pragma unroll
+    for (int j = 0; j < kRowE; ++j) {
+        const float add = (j == jT ? cw : 0.f) + (j == jST ? cws : 0.f);
+        dT[j] += add;
+        dR[j] += add;
+        dS[j] += j == jST ? cws : 0.f;
+    }
+    return make_float2(lT, lST);
+}
+
+template <int NL, int KP>
+__global__ void __launch_bounds__(32 * kRowWarps, 3) cache_loss_rows_kernel(const LossArgs a) {
+    constexpr int CPW = 32 / NL;                         // tasks per warp
+    const int lane = threadIdx.x & 31;
+    const int half = NL == 2 ? (lane & 1) : 0;
+    const int warp = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    const int BL = a.B * a.L;
+    const int wpc = (BL + CPW - 1) / CPW;                // warps per token chunk
+    if (warp >= wpc * a.nchunks) return;                 // whole warps
+    const int c = warp / wpc;
+    const int jl = (warp % wpc) * CPW + lane / NL;       // b * L + l
+    const bool active = jl < BL;                         // idle pairs run on zeros
+    const int T = a.T, L = a.L, N = a.N;
+    const int b = active ? jl / L : 0, l = active ? jl % L : 0;
+    const int t0 = c * a.chunk;
+    const int t1 = min(T, t0 + a.chunk);
+    const bool st = a.heads == 3;
+    const bool wr = active && a.grad != nullptr;
+    const size_t row3 = (size_t)3 * N;
+    const size_t tok = (size_t)L * row3;
+    const size_t base = ((size_t)b * T * L + l) * row3 + (size_t)half * kRowE;
+    const size_t s_off = l > 0 ? tok + (size_t)2 * N - row3 : (size_t)(L - 1 - l) * row3 + 2 * N;
+    const float* pp = a.probs + base + (size_t)t0 * tok;
+    float* gp = a.grad ? a.grad + base + (size_t)t0 * tok : nullptr;
+    float* lossp = (a.loss && active && half == 0)
+                       ? a.loss + (((size_t)b * T + t0) * L + l) * 2 : nullptr;
+
+    // The rows of step t are copied into shared memory one step ahead
+    // (cp.async, two stages); each warp's accesses to a stage are contiguous.
+    __shared__ RowStage stg[2];
+    const int x = threadIdx.x;
+    auto prefetch = [&](int k, const float* u, int t) {       // u: unit (b, t, l)
+        const bool nx = active && t + 1 < T;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) cp_async16(&stg[k][i][x], u + N + 4 * i, active);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) cp_async16(&stg[k][4 + i][x], nx ? u + tok + 4 * i : u, nx);
+        if (st) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                cp_async16(&stg[k][8 + i][x], nx ? u + s_off + 4 * i : u, nx);
+        }
+        cp_async_commit();
+    };
+    auto take_q = [&](float (&v)[kRowE], int k) {       // p^R_{t+1} of stage k
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float4 f = lds4(stg[k][4 + i][x]);
+            v[4 * i] = f.x;
+            v[4 * i + 1] = f.y;
+            v[4 * i + 2] = f.z;
+            v[4 * i + 3] = f.w;
+        }
+    };
+
+    float pR[kRowE], carry[kRowE];
+    float dR[kRowE], dT[kRowE], dS[kRowE];
+#pragma unroll
+    for (int j = 0; j < kRowE; ++j) carry[j] = 0.f;
+    double sumT = 0.0, sumST = 0.0;
+    prefetch(0, pp, t0);
+
+    if (t0 > 0) {
+        // halo: the terms of step t0 - 1 give the target part of p^R_{t0}
+        prefetch(1, pp - tok, t0 - 1);
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        load16(pR, pp - tok, active);
+        rows_step<NL, KP>(pR, stg[1], x, st, a.top_b, a, half, lane, carry, dR, dT, dS);
+        take_q(pR, 1);
+    } else {
+        load16(pR, pp, active);
+        if (lossp) lossp[1] = 0.f;                       // no l^ST at t = 0
+        if (st && wr && l > 0) {                         // p^S of rho(0, l) receives nothing
+            float z[kRowE];
+#pragma unroll
+            for (int j = 0; j < kRowE; ++j) z[j] = 0.f;
+            store16(gp + 2 * N - row3, z);
+        }
+    }
+
+#pragma unroll 1
+    for (int t = t0; t < t1; ++t, pp += tok) {
+        const int k = (t - t0) & 1;
+        if (t + 1 < t1)
+            prefetch(k ^ 1, pp + tok, t + 1);
+        else
+            cp_async_commit();                           // an empty group keeps the count
+        cp_async_wait1();                                // this step's copies have landed
+        const bool next = t + 1 < T;
+        if (next) {
+            const float2 y =
+                rows_step<NL, KP>(pR, stg[k], x, st, a.top_b, a, half, lane, carry, dR, dT, dS);
+            sumT += (double)y.x;
+            sumST += (double)y.y;
+            if (lossp) {
+                lossp[0] = y.x;
+                lossp[(size_t)L * 2 + 1] = st ? y.y : 0.f;
+            }
+        } else {
+            // last token: no l^T here, no l^ST after it
+            if (lossp) lossp[0] = 0.f;
+#pragma unroll
+            for (int j = 0; j < kRowE; ++j) {
+                dR[j] = carry[j];
+                dT[j] = dS[j] = 0.f;
+            }
+            if (st && wr && l == 0) {                    // p^S of rho(T, 0) receives nothing
+                float z[kRowE];
+#pragma unroll
+                for (int j = 0; j < kRowE; ++j) z[j] = 0.f;
+                store16(gp + s_off, z);
+            }
+        }
+        if (a.grad) {
+            // softmax backward of each head row: dz = p (dp - <p, dp>)
+            const bool ws = st && next;
+            float xR = 0.f, xT = 0.f, xS = 0.f;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float4 fT = lds4(stg[k][i][x]);
+                const float4 fS = ws ? lds4(stg[k][8 + i][x]) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    const int j = 4 * i + c;
+                    xR = fmaf(pR[j], dR[j], xR);
+                    xT = fmaf(f4(fT, c), dT[j], xT);
+                    xS = fmaf(f4(fS, c), dS[j], xS);
+                }
+            }
+            xR = pair_sum<NL>(xR);
+            xT = pair_sum<NL>(xT);
+            xS = pair_sum<NL>(xS);
+            if (wr) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int j = 4 * i;
+                    __stcs(reinterpret_cast<float4*>(gp) + i,
+                           make_float4(pR[j] * (dR[j] - xR), pR[j + 1] * (dR[j + 1] - xR),
+                                       pR[j + 2] * (dR[j + 2] - xR), pR[j + 3] * (dR[j + 3] - xR)));
+                    const float4 fT = lds4(stg[k][i][x]);
+                    __stcs(reinterpret_cast<float4*>(gp + N) + i,
+                           make_float4(fT.x * (dT[j] - xT), fT.y * (dT[j + 1] - xT),
+                                       fT.z * (dT[j + 2] - xT), fT.w * (dT[j + 3] - xT)));
+                    if (ws) {
+                        const float4 fS = lds4(stg[k][8 + i][x]);
+                        __stcs(reinterpret_cast<float4*>(gp + s_off) + i,
+                               make_float4(fS.x * (dS[j] - xS), fS.y * (dS[j + 1] - xS),
+                                           fS.z * (dS[j + 2] - xS), fS.w * (dS[j + 3] - xS)));
+                    }
+                }
+            }
+            gp += tok;
+        }
+        if (lossp) lossp += (size_t)L * 2;
+        if (next) take_q(pR, k);
+    }
+    if (a.partial && active && half == 0) {
+        const size_t task = ((size_t)b * a.nchunks + c) * L + l;
+        a.partial[task * 2 + 0] = sumT;
+        a.partial[task * 2 + 1] = sumST;
+    }
+}
+
+// Token chunks of the short-row kernel: as many as give every resident warp
+// one (a single wave, each warp running one chunk of its 32 / NL chains),
+// chunks of at least 32 tokens so the halo step costs <= 1/32.
+template <int NL, int KP>
+int launch_loss_rows(LossArgs& a, cudaStream_t stream) {
+    constexpr int CPW = 32 / NL;
+    static std::atomic<int> blocks_per_sm{0};
+    if (blocks_per_sm.load() == 0) {
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, cache_loss_rows_kernel<NL, KP>,
+                                                          32 * kRowWarps, 0) != cudaSuccess)
+            return CRC_ECUDA;
+        blocks_per_sm.store(n > 0 ? n : 1);
+    }
+    const long long groups = (a.B * (long long)a.L + CPW - 1) / CPW;
+    const long long resident = (long long)sm_count() * blocks_per_sm.load() * kRowWarps;
+    long long n = resident / groups;
+    const long long cap = (a.T + 31) / 32;
+    if (n > cap) n = cap;
+    if (n < 1) n = 1;
+    a.chunk = (int)((a.T + n - 1) / n);
+    a.nchunks = (a.T + a.chunk - 1) / a.chunk;
+    const long long warps = groups * a.nchunks;
+    const int grid = (int)((warps + kRowWarps - 1) / kRowWarps);
+    {
+        ProfScope prof(CRC_KERNEL_LOSS, stream);
+        cache_loss_rows_kernel<NL, KP><<<grid, 32 * kRowWarps, 0, stream>>>(a);
+    }
+    note_launch();
+    return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
+}
+
+template <int NL>
+int launch_loss_rows_kp(LossArgs& a, cudaStream_t stream) {
+    if (a.top_b <= 2) return launch_loss_rows<NL, 2>(a, stream);
+    if (a.top_b <= 4) return launch_loss_rows<NL, 4>(a, stream);
+    if (a.top_b <= 8) return launch_loss_rows<NL, 8>(a, stream);
+    return launch_loss_rows<NL, 16>(a, stream);
+}
+
 // Means L_T, L_ST: fixed-order sums of the per-task sums (deterministic).
 constexpr int kMeanThreads = 256;
 
@@ -514,6 +926,13 @@ int launch_loss_t(const LossArgs& a, cudaStream_t stream) {
 }
 
 }  // namespace
+
+long long loss_task_slots(int B, int L, int T, int N) {
+    const long long bl = (long long)B * L;
+    if (T <= 0) return 0;
+    if (N <= 32) return bl * ((T + 31) / 32);
+    return bl * loss_plan(B, L, T).nchunks;
+}
 
 LossPlan loss_plan(int B, int L, int T) {
     // About 49152 warp tasks (ten waves of resident warps on a 152-SM GPU,
@@ -557,6 +976,10 @@ int launch_cache_loss(const crc_problem& p, const float* probs, int T, int heads
     a.gT = (float)(cT / tau);
     a.gST = (float)(cST / tau);
     int rc;
+    if ((p.N == 16 || p.N == 32) && top_b <= 16) {
+        // short rows: 16 elements per lane, one or two lanes per row
+        rc = p.N == 16 ? launch_loss_rows_kp<1>(a, stream) : launch_loss_rows_kp<2>(a, stream);
+    } else {
 #define CRC_LOSS_V(VV)                                                               \
     rc = p.N == 32 * VV ? launch_loss_t<VV, true>(a, stream)                         \
                         : launch_loss_t<VV, false>(a, stream);
@@ -570,12 +993,13 @@ int launch_cache_loss(const crc_problem& p, const float* probs, int T, int heads
         CRC_LOSS_V(8)
     }
 #undef CRC_LOSS_V
+    }
     if (rc != CRC_OK || !means) return rc;
     const double inv_n = n_valid > 0 ? 1.0 / n_valid : 0.0;
     {
         ProfScope prof(CRC_KERNEL_LOSS_MEANS, stream);
         loss_means_kernel<<<1, kMeanThreads, 0, stream>>>(
-            static_cast<const double*>(workspace), p.B * p.L * pl.nchunks, inv_n,
+            static_cast<const double*>(workspace), p.B * p.L * a.nchunks, inv_n,
             heads == 3 ? inv_n : 0.0, means);
     }
     note_launch();

@@ -81,6 +81,15 @@ CASES = [  # name, B, T, L, N, top_b, tau, quant
     ("ties_n128", 2, 30, 2, 128, 20, 0.03, 64),
     ("b1", 2, 30, 2, 128, 1, 0.03, None),
     ("bN", 1, 30, 2, 32, 32, 0.05, None),
+    # short rows (N = 16, 32 with top_b <= 16): one or two lanes per row
+    ("n32_ties", 2, 40, 3, 32, 8, 0.05, 16),
+    ("n32_ties_fine", 2, 40, 3, 32, 6, 0.05, 256),
+    ("n32_b16", 2, 40, 3, 32, 16, 0.05, None),
+    ("n32_b1", 2, 30, 2, 32, 1, 0.05, None),
+    ("n32_b3", 3, 33, 5, 32, 3, 0.1, None),
+    ("n32_b17", 1, 30, 2, 32, 17, 0.05, None),
+    ("n16_ties", 2, 40, 3, 16, 5, 0.05, 8),
+    ("n16_b16", 2, 30, 2, 16, 16, 0.05, None),
 ]
 
 
@@ -90,16 +99,19 @@ def test_loss_and_gradient_match_oracle(C, oracle_lib, name, B, T, L, N, top_b, 
     check(C, oracle_lib, p32, top_b, tau, w_T=0.7, w_ST=1.3)
 
 
+@pytest.mark.parametrize("N,top_b", [(128, 20), (32, 8)])
 @pytest.mark.parametrize("kind", ["uncorrelated", "repeated", "repeated_ties"])
-def test_theta_guess_extremes(C, oracle_lib, kind):
+def test_theta_guess_extremes(C, oracle_lib, kind, N, top_b):
     """theta_B starts from the previous token's: far off when consecutive
-    tokens are unrelated, exact when they repeat (with ties at theta too)."""
+    tokens are unrelated, exact when they repeat (with ties at theta too).
+    N = 32 runs the short-row kernel on the same extremes."""
     if kind == "uncorrelated":
-        p32 = S.distributions(2, 60, 3, 128, seed=13, rho=0.0)
+        p32 = S.distributions(2, 60, 3, N, seed=13, rho=0.0)
     else:
-        p32 = np.repeat(S.distributions(2, 1, 3, 128, seed=14,
-                                        quant=64 if kind == "repeated_ties" else None), 50, axis=1)
-    check(C, oracle_lib, np.ascontiguousarray(p32), 20, 0.03)
+        p32 = np.repeat(S.distributions(2, 1, 3, N, seed=14,
+                                        quant=N // 2 if kind == "repeated_ties" else None), 50,
+                        axis=1)
+    check(C, oracle_lib, np.ascontiguousarray(p32), top_b, 0.03)
 
 
 @pytest.mark.parametrize("w_T,w_ST", [(0.0, 1.0), (1.0, 0.0), (0.1, 0.0)])
@@ -109,19 +121,20 @@ def test_objective_weights(C, oracle_lib, w_T, w_ST):
     check(C, oracle_lib, p32, 20, 0.03, w_T, w_ST)
 
 
-def test_update_only_heads_2(C, oracle_lib):
+@pytest.mark.parametrize("N,top_b", [(128, 20), (32, 8)])
+def test_update_only_heads_2(C, oracle_lib, N, top_b):
     """heads = 2 never reads the S head (NaN here) and leaves its gradient rows."""
-    p32 = S.distributions(2, 45, 3, 128, seed=8)
-    check(C, oracle_lib, p32, 20, 0.03, heads=2)
+    p32 = S.distributions(2, 45, 3, N, seed=8)
+    check(C, oracle_lib, p32, top_b, 0.03, heads=2)
     nan_s = p32.copy()
     nan_s[..., 2, :] = np.nan
-    pr = problem(C, 2, 3, 128)
+    pr = problem(C, 2, 3, N)
     probs = torch.from_numpy(nan_s).cuda()
     grad = torch.full(probs.shape, 7.0, device="cuda")
-    loss, means, _ = C.cache_loss(pr, probs, 20, 0.03, heads=2, grad_out=grad)
+    loss, means, _ = C.cache_loss(pr, probs, top_b, 0.03, heads=2, grad_out=grad)
     g = grad.cpu().numpy()
     assert np.all(g[..., 2, :] == 7.0)
-    ref = run(C, p32, 20, 0.03, heads=2)
+    ref = run(C, p32, top_b, 0.03, heads=2)
     assert np.array_equal(loss.cpu().numpy(), ref[0])
     assert np.array_equal(g[..., :2, :], ref[2][..., :2, :])
 
@@ -134,25 +147,28 @@ def test_short_sequences(C, oracle_lib, T):
         assert np.all(loss == 0) and np.all(means == 0) and np.all(g == 0)
 
 
-def test_chunks_and_halos(C, oracle_lib):
+@pytest.mark.parametrize("N,top_b", [(128, 20), (32, 8)])
+def test_chunks_and_halos(C, oracle_lib, N, top_b):
     """One stream over two layers splits its tokens into chunks, each with a
     halo step.  T = 300 makes 10 chunks of 30 tokens; the first 250 tokens
     alone make 8 chunks of 32, and give the same values wherever the two
-    sequences see the same neighbours (the coefficients matched)."""
-    p32 = S.distributions(1, 300, 2, 128, seed=9)
-    la, _, ga = check(C, oracle_lib, p32, 20, 0.03)
+    sequences see the same neighbours (the coefficients matched).  At N = 32
+    the two chains of a chunk share a warp with 14 idle row pairs."""
+    p32 = S.distributions(1, 300, 2, N, seed=9)
+    la, _, ga = check(C, oracle_lib, p32, top_b, 0.03)
     w = 249 / 299                                          # same w / (B (T - 1) L)
-    lb, _, gb = run(C, np.ascontiguousarray(p32[:, :250]), 20, 0.03, w_T=w, w_ST=w)
+    lb, _, gb = run(C, np.ascontiguousarray(p32[:, :250]), top_b, 0.03, w_T=w, w_ST=w)
     assert np.array_equal(la[:, :249, :, 0], lb[:, :249, :, 0])
     assert np.array_equal(la[:, :250, :, 1], lb[:, :250, :, 1])
     np.testing.assert_allclose(gb[:, :249], ga[:, :249], rtol=1e-6, atol=1e-12)
 
 
-def test_forward_only_and_determinism(C):
-    p32 = S.distributions(4, 80, 6, 128, seed=10)
-    l1, m1, g1 = run(C, p32, 20, 0.03)
-    l2, m2, g2 = run(C, p32, 20, 0.03)
-    l3, m3, _ = run(C, p32, 20, 0.03, grad=False)
+@pytest.mark.parametrize("N,top_b", [(128, 20), (32, 8)])
+def test_forward_only_and_determinism(C, N, top_b):
+    p32 = S.distributions(4, 80, 6, N, seed=10)
+    l1, m1, g1 = run(C, p32, top_b, 0.03)
+    l2, m2, g2 = run(C, p32, top_b, 0.03)
+    l3, m3, _ = run(C, p32, top_b, 0.03, grad=False)
     assert np.array_equal(l1, l2) and np.array_equal(m1, m2) and np.array_equal(g1, g2)
     assert np.array_equal(l1, l3) and np.array_equal(m1, m3)
 
