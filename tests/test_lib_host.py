@@ -162,6 +162,10 @@ def test_cache_loss_argument_checks(crc):
     # per-task fp64 sums: B * L tasks per token chunk, 16 chunks of 64 tokens at T = 1024
     assert crc.crc_loss_workspace_bytes(p, 1024) == 64 * 48 * 16 * 16
     assert crc.crc_loss_workspace_bytes(p, 0) == 0
+    # N <= 32: chunks are sized at launch, so one slot per stream, layer and 32 tokens
+    g = crc.problem_of(S.GPT_OSS_20B)
+    assert crc.crc_loss_workspace_bytes(g, 2048) == 128 * 24 * 64 * 16
+    assert crc.crc_loss_workspace_bytes(g, 33) == 128 * 24 * 2 * 16
     ws = crc.crc_loss_workspace_bytes(p, 8)
     call = lambda T=8, heads=3, top_b=20, tau=0.03, wT=1.0, wST=1.0, probs=256, loss=256, \
         means=None, grad=None, ws_ptr=256, ws_bytes=ws: lib.crc_cache_loss(  # noqa: E731
