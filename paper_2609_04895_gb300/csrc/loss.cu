@@ -1,5 +1,6 @@
 // Soft Top-B cache-coverage losses and their gradient (Sec. 3.1-3.4), from the
-// router probabilities, one warp per (stream, layer, token chunk).
+// router probabilities: one warp per (stream, layer, token chunk), or for
+// short rows (N = 16, 32 with top_b <= 16) one or two lanes per such task.
 //
 // For a priority s over N experts and a target distribution q:
 //   theta_B(s) = the B-th largest entry of s,
