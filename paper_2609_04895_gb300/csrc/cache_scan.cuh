@@ -361,9 +361,14 @@ __device__ __forceinline__ void row_topk_mask(const float* row, int N, int K, ui
 // loop it would meet a cache whose lowest member is no lower than it and lose
 // the strict test, ending the pass exactly as the rank test or the strict
 // test ends it here.
+//
+// With nD_out, the first rank count also carries this lane's demand misses of
+// `sel` against the cache as it stands; when that count ends the pass (the
+// cache unchanged), *nD_out receives the warp's demand misses, else -1.
 template <int V, bool ALL_VALID>
 __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V], uint32_t valid,
-                                           int lane, int C, int R) {
+                                           int lane, int C, int R, uint32_t sel = 0u,
+                                           int* nD_out = nullptr) {
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
     uint32_t kS[V];
 #pragma unroll
@@ -371,9 +376,10 @@ __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V
         kS[v] = is_valid(v) ? pkey(__fadd_rn(cr.aT[v], pS[v])) : 0u;
     uint32_t left = valid & ~cr.cache;         // non-residents not yet taken
     int pro = 0;
+    if (nD_out) *nD_out = -1;
 #pragma unroll 1
     for (int j = 0; j < R; ++j) {
-        // the best remaining non-resident: largest key, then lowest index
+        // the best remaining non-resident c: largest key, then lowest index
         uint32_t m[V];
 #pragma unroll
         for (int v = 0; v < V; ++v) m[v] = ((left >> v) & 1u) ? kS[v] : 0u;
@@ -382,22 +388,30 @@ __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V
         for (int v = 1; v < V; ++v) best = umax(best, m[v]);
         const uint32_t mx = __reduce_max_sync(kFull, best);
         if (mx == 0u) break;                   // no non-resident left
-        const int owner = __ffs(__ballot_sync(kFull, best == mx)) - 1;
-        uint32_t cs = 0u;
-#pragma unroll
-        for (int v = V - 1; v >= 0; --v) cs = m[v] == mx ? (uint32_t)v : cs;   // lowest such slot
         // rank of c: experts with higher keys, and with equal keys at lower
         // indices (lanes before the owner; the owner's slots before c's).
-        // Invalid slots hold key 0 and count for neither.
+        // Invalid slots hold key 0 and count for neither.  Fields of 9 bits
+        // (counts <= N <= 256), the demand misses above them.
         uint32_t gt = 0u, eq = 0u;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
             gt += kS[v] > mx ? 1u : 0u;
             eq += kS[v] == mx ? 1u : 0u;
         }
-        const uint32_t tot = __reduce_add_sync(kFull, gt | (eq << 16));
-        uint32_t rank = tot & 0xffffu;
-        if ((tot >> 16) > 1u) {                // c shares its key: count those before it by index
+        uint32_t packed = gt | (eq << 9);
+        if (nD_out && j == 0) packed |= (uint32_t)__popc(sel & ~cr.cache) << 18;
+        const uint32_t tot = __reduce_add_sync(kFull, packed);
+        uint32_t rank = tot & 0x1ffu;
+        const bool tie = ((tot >> 9) & 0x1ffu) > 1u;   // c shares its key
+        int owner = 0;
+        uint32_t cs = 0u;
+        auto locate = [&]() {                  // c's lane and slot
+            owner = __ffs(__ballot_sync(kFull, best == mx)) - 1;
+#pragma unroll
+            for (int v = V - 1; v >= 0; --v) cs = m[v] == mx ? (uint32_t)v : cs;   // lowest slot
+        };
+        if (tie) {                             // count those before c by index
+            locate();
             const uint32_t c_slot = __shfl_sync(kFull, cs, owner);
             uint32_t before = 0u;
 #pragma unroll
@@ -406,7 +420,11 @@ __device__ __forceinline__ int scan_refine(ChainRegs<V>& cr, const float (&pS)[V
                               ? 1u : 0u;
             rank += __reduce_add_sync(kFull, before);
         }
-        if ((int)rank >= R) break;             // c is not among the top R, nor is any later one
+        if ((int)rank >= R) {                  // c is not among the top R, nor is any later one
+            if (nD_out && j == 0) *nD_out = (int)(tot >> 18);
+            break;
+        }
+        if (!tie) locate();
         const uint32_t cbit = (lane == owner) ? (1u << cs) : 0u;
         left &= ~cbit;
         if (cr.count < C) {                    // free slot: proactive load
@@ -437,11 +455,12 @@ __device__ __forceinline__ int scan_apply(ChainRegs<V>& cr, const float (&sT)[V]
                                           const float (&pS)[V], bool refine, uint32_t valid,
                                           int lane, int K, int C, int R, uint32_t sel,
                                           int* n_miss) {
-    int pro = refine ? scan_refine<V, ALL_VALID>(cr, pS, valid, lane, C, R) : 0;
+    int nD_pre = -1;
+    int pro = refine ? scan_refine<V, ALL_VALID>(cr, pS, valid, lane, C, R, sel, &nD_pre) : 0;
 
     // demand misses and UpdateCache (Algorithm 1)
     const uint32_t dem = sel & ~cr.cache;
-    const int nD = (int)__reduce_add_sync(kFull, (uint32_t)__popc(dem));
+    const int nD = nD_pre >= 0 ? nD_pre : (int)__reduce_add_sync(kFull, (uint32_t)__popc(dem));
     const int freeslots = C - cr.count;
     if (nD > freeslots) {
         uint32_t kT[V];
@@ -576,6 +595,7 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
     const uint32_t parity = hdr->parity;
 
     uint32_t* err = &hdr->error;
+    (void)err;                                  // read only by the checking build's bounds checks
     if (active && hdr_ok && CRC_IN_BOUNDS(a.trace_t0 >= 0 && a.trace_t0 + a.T <= a.trace_T, err)) {
         const int b = chain / a.L, l = chain % a.L;
         const int N = a.N, L = a.L, T = a.T;
