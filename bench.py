@@ -231,7 +231,9 @@ KERNEL_SOURCES = {
               "crc_device.cuh"],
     "router": ["router.cu", "router_gemm.cuh", "crc_device.cuh"],
     "scan": ["scan.cu", "cache_scan.cuh", "crc_device.cuh"],
-    "policy": ["policy.cu", "policy_scan.cuh", "cache_scan.cuh", "crc_device.cuh"],
+    "policy": ["policy.cu", "policy_launch.cuh", "policy_lru.cu", "policy_lfu.cu",
+               "policy_lrfu.cu", "policy_spatio.cu", "policy_scan.cuh", "cache_scan.cuh",
+               "crc_device.cuh"],
     "loss": ["loss.cu", "cache_scan.cuh", "crc_device.cuh"],
 }
 

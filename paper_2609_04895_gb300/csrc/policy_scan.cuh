@@ -39,10 +39,12 @@ __device__ __forceinline__ float lrfu_decay(int lambda2, uint32_t dt) {
     return f;
 }
 
-// One access of the chain at token t under the policy.  aux: this lane's
-// integer priorities (LRU, Spatio-only, LRFU: token of last use; LFU: count);
-// cr.aT: the float ones (LRFU: CRF; Spatio-only: p^R of the previous token).
-template <int V, bool ALL_VALID>
+// One access of the chain at token t under the policy POL (a CRC_POLICY_*
+// value, fixed at compile time so that each policy's step carries only its
+// own priority arithmetic).  aux: this lane's integer priorities (LRU,
+// Spatio-only, LRFU: token of last use; LFU: count); cr.aT: the float ones
+// (LRFU: CRF; Spatio-only: p^R of the previous token).
+template <int V, bool ALL_VALID, int POL>
 __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V],
                                             const float (&pR)[V], const float (&pS)[V],
                                             bool refine, uint32_t valid, int lane,
@@ -52,7 +54,7 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
     auto is_valid = [&](int v) { return ALL_VALID || ((valid >> v) & 1u); };
     const int K = a.s.K, C = a.s.C;
     int pro = 0;
-    if (a.policy == CRC_POLICY_SPATIO_LRU && refine) {
+    if (POL == CRC_POLICY_SPATIO_LRU && refine) {
         const uint32_t before = cr.cache;
         pro = scan_refine<V, ALL_VALID>(cr, pS, valid, lane, C, a.s.R);
         const uint32_t loaded = cr.cache & ~before;
@@ -93,7 +95,7 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
         uint32_t kV[V];
 #pragma unroll
         for (int v = 0; v < V; ++v)
-            kV[v] = a.policy == CRC_POLICY_LRFU
+            kV[v] = POL == CRC_POLICY_LRFU
                         ? __float_as_uint(__fmul_rn(cr.aT[v], lrfu_decay(a.lambda2, t - aux[v])))
                         : aux[v];
         uint32_t vset = cr.cache & ~sel;
@@ -114,9 +116,9 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
     for (int v = 0; v < V; ++v) {
         if (!((sel >> v) & 1u)) continue;
         const bool h = (hit >> v) & 1u;
-        if (a.policy == CRC_POLICY_LFU) {
+        if constexpr (POL == CRC_POLICY_LFU) {
             aux[v] = h ? aux[v] + 1u : 1u;
-        } else if (a.policy == CRC_POLICY_LRFU) {
+        } else if constexpr (POL == CRC_POLICY_LRFU) {
             cr.aT[v] = h ? __fadd_rn(1.f, __fmul_rn(lrfu_decay(a.lambda2, t - aux[v]), cr.aT[v]))
                          : 1.f;
             aux[v] = t;
@@ -124,7 +126,7 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
             aux[v] = t;
         }
     }
-    if (a.policy == CRC_POLICY_SPATIO_LRU) {
+    if constexpr (POL == CRC_POLICY_SPATIO_LRU) {
 #pragma unroll
         for (int v = 0; v < V; ++v) cr.aT[v] = pR[v];            // p^R_{t-1} for the next access
     }
@@ -138,7 +140,7 @@ __device__ __forceinline__ void policy_step(ChainRegs<V>& cr, uint32_t (&aux)[V]
     }
 }
 
-template <int V, bool ALL_VALID, int KP>
+template <int V, bool ALL_VALID, int KP, int POL>
 __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWarps)
     cache_scan_policy_kernel(PolicyArgs pa) {
     // Top-K sets of the next 32 tokens of each warp's chain, one row per token
@@ -196,7 +198,7 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
             if (t > 0) return unit_ptr(t - 1, L - 1) + 2 * N;
             return carry_in;
         };
-        const bool want_s = pa.policy == CRC_POLICY_SPATIO_LRU && a.R > 0;
+        const bool want_s = POL == CRC_POLICY_SPATIO_LRU && a.R > 0;
         // without a rank-order trace the Top-K set is taken for 32 tokens at
         // a time, lane j for token t + j (it does not depend on the cache)
         const bool batch_sel = a.trace_topk == nullptr;
@@ -233,15 +235,15 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
             const bool refine = want_s && (t0 + t >= 1);
             if (traced) {
                 const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
-                policy_step<V, ALL_VALID>(cr, aux, cR.v, cS.v, refine, valid, lane, pa,
-                                          (uint32_t)(t0 + t), batch_sel, sel_in,
+                policy_step<V, ALL_VALID, POL>(cr, aux, cR.v, cS.v, refine, valid, lane, pa,
+                                               (uint32_t)(t0 + t), batch_sel, sel_in,
                                           a.trace_topk ? a.trace_topk + unit * a.K : nullptr,
                                           a.trace_miss ? a.trace_miss + unit : nullptr,
                                           a.trace_pro ? a.trace_pro + unit : nullptr);
             } else {
-                policy_step<V, ALL_VALID>(cr, aux, cR.v, cS.v, refine, valid, lane, pa,
-                                          (uint32_t)(t0 + t), true, sel_in, nullptr, nullptr,
-                                          nullptr);
+                policy_step<V, ALL_VALID, POL>(cr, aux, cR.v, cS.v, refine, valid, lane, pa,
+                                               (uint32_t)(t0 + t), true, sel_in, nullptr,
+                                               nullptr, nullptr);
             }
             cR = nR;
             cS = nS;
