@@ -230,7 +230,7 @@ KERNEL_SOURCES = {
               "fused_n64.cu", "fused_n128.cu", "router_gemm.cuh", "cache_scan.cuh",
               "crc_device.cuh"],
     "router": ["router.cu", "router_gemm.cuh", "crc_device.cuh"],
-    "scan": ["scan.cu", "cache_scan.cuh", "crc_device.cuh"],
+    "scan": ["scan.cu", "scan_traced.cu", "scan_launch.cuh", "cache_scan.cuh", "crc_device.cuh"],
     "policy": ["policy.cu", "policy_launch.cuh", "policy_lru.cu", "policy_lfu.cu",
                "policy_lrfu.cu", "policy_spatio.cu", "policy_scan.cuh", "cache_scan.cuh",
                "crc_device.cuh"],

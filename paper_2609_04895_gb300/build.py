@@ -17,7 +17,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libcrc.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-UNITS = ["api.cu", "router.cu", "scan.cu", "synth.cu", "noalloc.cu", "fused.cu",
+UNITS = ["api.cu", "router.cu", "scan.cu", "scan_traced.cu", "synth.cu", "noalloc.cu", "fused.cu",
          "fused_n16.cu", "fused_n32.cu", "fused_n64.cu", "fused_n128.cu", "policy.cu",
          "policy_lru.cu", "policy_lfu.cu", "policy_lrfu.cu", "policy_spatio.cu", "loss.cu",
          "transfer.cu", "probe.cu"]

@@ -573,7 +573,9 @@ __device__ __forceinline__ uint32_t lane_bits(const uint32_t* words, int lane, i
 // four put 24 on some SMs and 20 on the rest).
 constexpr int kScanWarps = 1;
 
-template <int V, bool ALL_VALID, int KP>
+// TRACED: compiled with the trace writes (any trace array given); the
+// untraced kernel carries none of their code.
+template <int V, bool ALL_VALID, int KP, bool TRACED>
 __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWarps)
     cache_scan_kernel(ScanArgs a) {
     // Top-K sets of the next 32 tokens of each warp's chain, one row per token
@@ -635,7 +637,7 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
 
         // Without a trace only the Top-K *set* is needed: it does not depend on
         // the cache, so lane j computes it for token t + j ahead of the chain.
-        const bool batch_sel = a.trace_topk == nullptr;
+        const bool batch_sel = !TRACED || a.trace_topk == nullptr;
         uint32_t (*sel_rows)[8] = sel_s[(threadIdx.x >> 5) % kScanWarps];
         const float* row_base = a.scores + ((size_t)b * T * L + l) * row;   // token 0 of chain
         // running pointer to this lane's part of unit (b, t, l); p^S of rho(t, l)
@@ -645,8 +647,6 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
                                       : (ptrdiff_t)(L - 1) * (ptrdiff_t)row - (ptrdiff_t)tok +
                                             (ptrdiff_t)2 * N;
         const float* up = unit_ptr(0, l);
-        const bool traced = a.trace_topk || a.trace_miss || a.trace_pro || a.trace_mid ||
-                            a.trace_after || a.trace_sel;
 
         Vec<V> cR = load_vec<V>(unit_ptr(0, l), has && unit_ok(0, l));
         Vec<V> cT = load_vec<V>(unit_ptr(0, l) + N, has && unit_ok(0, l));
@@ -678,7 +678,7 @@ __global__ void __launch_bounds__(32 * kScanWarps, (V >= 8 ? 12 : 24) / kScanWar
             }
             up += tok;
             const bool refine = want_s && (t0 + t >= 1);
-            if (traced) {
+            if constexpr (TRACED) {
                 const size_t unit = ((size_t)b * a.trace_T + a.trace_t0 + t) * L + l;
                 const size_t NWs = (size_t)((N + 31) >> 5);
                 scan_step<V, ALL_VALID>(cr, cR.v, cT.v, cS.v, refine, valid, lane, a.K, a.C, a.R,
