@@ -178,7 +178,7 @@ __device__ __forceinline__ void ring_vec(const uint8_t* base, int lane, int r, f
 // is complete when `publishers` epilogue warps have published it), runs
 // Algorithm 2 / 1 on each token (scan_apply) and releases the tiles through
 // the monotonic reader counters.
-template <int NH, int V, bool ALL_VALID>
+template <int NH, int V, bool ALL_VALID, bool TRACED>
 __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* err,
                                                 uint32_t* abort_flag, int64_t t0g,
                                                 uint32_t parity, int lane, uint32_t publishers) {
@@ -196,7 +196,7 @@ __device__ __forceinline__ void fused_scan_role(const FusedArgs& a, uint32_t* er
     const bool want_s = a.R > 0;
     const uint32_t e0 = (uint32_t)lane * V;
     const int NW = (N + 31) >> 5;
-    const bool traced = a.tr_miss || a.tr_pro || a.tr_mid || a.tr_after || a.tr_sel;
+    const bool traced = TRACED && (a.tr_miss || a.tr_pro || a.tr_mid || a.tr_after || a.tr_sel);
     while (true) {
         uint32_t item = 0u;
         if (lane == 0) item = atomicAdd(&a.ctl[0], 1u);
@@ -417,7 +417,8 @@ struct FusedCfg {
                   "swizzle atom alignment");
 };
 
-template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR = false>
+// TRACED: compiled with the scan role's trace writes (any trace array given).
+template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR = false, bool TRACED = false>
 __global__ void __launch_bounds__(512, 1)
     fused_route_cache_kernel(const __grid_constant__ CUtensorMap tmap_h,
                              const __grid_constant__ CUtensorMap tmap_w, FusedArgs a) {
@@ -915,7 +916,7 @@ __global__ void __launch_bounds__(512, 1)
             if (!ok) break;
         }
     } else if (hdr_ok) {
-        fused_scan_role<NH, V, ALL_VALID>(a, err, abort_flag, t0g, parity, lane, 4u);
+        fused_scan_role<NH, V, ALL_VALID, TRACED>(a, err, abort_flag, t0g, parity, lane, 4u);
     }
     tc_fence_before();
     __syncthreads();

@@ -54,7 +54,7 @@ inline FusedPlan fused_plan(const crc_problem& p, int T) {
 // PAIR launches clusters of two CTAs (the GEMM on CTA pairs), cooperatively so
 // that every CTA is resident; a device that refuses that launch gets the
 // single-CTA kernel from then on (CRC_EUNSUPPORTED).
-template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR = false>
+template <int NH, int H, int V, bool ALL_VALID, int KP, bool PAIR, bool TRACED>
 int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                    void* state, void* workspace, const crc_trace* trace,
                       cudaStream_t stream) {
@@ -62,7 +62,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
     using RC = typename Cfg::RC;
     const FusedPlan f = fused_plan(p, T);
     if (PAIR && (f.SB != 1 || f.n_bg % 2 != 0)) return CRC_EUNSUPPORTED;
-    auto kern = fused_route_cache_kernel<NH, H, V, ALL_VALID, KP, PAIR>;
+    auto kern = fused_route_cache_kernel<NH, H, V, ALL_VALID, KP, PAIR, TRACED>;
     // -1: not set up yet in this process; 0: refused; else the grid
     static int grid = -1;
     if (grid == 0) return CRC_EUNSUPPORTED;
@@ -182,7 +182,7 @@ int launch_fused_t(const crc_problem& p, const uint16_t* hidden, const uint16_t*
 
 // The GEMM on CTA pairs (N = 128: three heads, or two in update-only mode)
 // when the tiles pair up; CRC_EUNSUPPORTED sends the call to one CTA per tile.
-template <int NH, int H, int V, bool ALL_VALID>
+template <int NH, int H, int V, bool ALL_VALID, bool TRACED>
 int launch_fused_pair(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat, int T,
                       void* state, void* workspace, const crc_trace* trace,
                       cudaStream_t stream) {
@@ -190,38 +190,42 @@ int launch_fused_pair(const crc_problem& p, const uint16_t* hidden, const uint16
         return CRC_EUNSUPPORTED;
     } else {
         if (p.K <= 2)
-            return launch_fused_t<NH, H, V, ALL_VALID, 2, true>(p, hidden, w_cat, T, state,
-                                                                workspace, trace, stream);
+            return launch_fused_t<NH, H, V, ALL_VALID, 2, true, TRACED>(p, hidden, w_cat, T,
+                                                                        state, workspace, trace,
+                                                                        stream);
         if (p.K <= 4)
-            return launch_fused_t<NH, H, V, ALL_VALID, 4, true>(p, hidden, w_cat, T, state,
-                                                                workspace, trace, stream);
+            return launch_fused_t<NH, H, V, ALL_VALID, 4, true, TRACED>(p, hidden, w_cat, T,
+                                                                        state, workspace, trace,
+                                                                        stream);
         if (p.K <= 8)
-            return launch_fused_t<NH, H, V, ALL_VALID, 8, true>(p, hidden, w_cat, T, state,
-                                                                workspace, trace, stream);
+            return launch_fused_t<NH, H, V, ALL_VALID, 8, true, TRACED>(p, hidden, w_cat, T,
+                                                                        state, workspace, trace,
+                                                                        stream);
         return CRC_EUNSUPPORTED;
     }
 }
 
 // Dispatch on heads (R > 0 needs the Spatio head) and the Top-K network width.
-template <int NH, int V, bool ALL_VALID>
-int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat,
+template <int NH, int V, bool ALL_VALID, bool TRACED>
+int launch_fused_mode(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat,
                        int T, void* state, void* workspace, const crc_trace* trace,
                        cudaStream_t stream) {
 #define CRC_FUSED_KP(HV)                                                                      \
     {                                                                                         \
-        const int rc = launch_fused_pair<NH, HV, V, ALL_VALID>(p, hidden, w_cat, T, state,    \
-                                                               workspace, trace, stream);     \
+        const int rc = launch_fused_pair<NH, HV, V, ALL_VALID, TRACED>(p, hidden, w_cat, T,   \
+                                                                       state, workspace,      \
+                                                                       trace, stream);        \
         if (rc != CRC_EUNSUPPORTED) return rc;                                                \
     }                                                                                         \
     if (p.K <= 2)                                                                             \
-        return launch_fused_t<NH, HV, V, ALL_VALID, 2>(p, hidden, w_cat, T, state, workspace, \
-                                                       trace, stream);                        \
+        return launch_fused_t<NH, HV, V, ALL_VALID, 2, false, TRACED>(                        \
+            p, hidden, w_cat, T, state, workspace, trace, stream);                            \
     if (p.K <= 4)                                                                             \
-        return launch_fused_t<NH, HV, V, ALL_VALID, 4>(p, hidden, w_cat, T, state, workspace, \
-                                                       trace, stream);                        \
+        return launch_fused_t<NH, HV, V, ALL_VALID, 4, false, TRACED>(                        \
+            p, hidden, w_cat, T, state, workspace, trace, stream);                            \
     if (p.K <= 8)                                                                             \
-        return launch_fused_t<NH, HV, V, ALL_VALID, 8>(p, hidden, w_cat, T, state, workspace, \
-                                                       trace, stream);                        \
+        return launch_fused_t<NH, HV, V, ALL_VALID, 8, false, TRACED>(                        \
+            p, hidden, w_cat, T, state, workspace, trace, stream);                            \
     return CRC_EUNSUPPORTED;
     if (p.R > 0) {
         CRC_FUSED_KP(3)
@@ -229,6 +233,20 @@ int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint1
         CRC_FUSED_KP(2)
     }
 #undef CRC_FUSED_KP
+}
+
+// The kernel without trace writes unless the call asks for a trace array.
+template <int NH, int V, bool ALL_VALID>
+int launch_fused_for_n(const crc_problem& p, const uint16_t* hidden, const uint16_t* w_cat,
+                       int T, void* state, void* workspace, const crc_trace* trace,
+                       cudaStream_t stream) {
+    const bool traced = trace && (trace->misses_dev || trace->proactive_dev ||
+                                  trace->cache_mid_dev || trace->cache_after_dev ||
+                                  trace->topk_set_dev);
+    return traced ? launch_fused_mode<NH, V, ALL_VALID, true>(p, hidden, w_cat, T, state,
+                                                              workspace, trace, stream)
+                  : launch_fused_mode<NH, V, ALL_VALID, false>(p, hidden, w_cat, T, state,
+                                                               workspace, nullptr, stream);
 }
 
 }  // namespace crc
