@@ -367,7 +367,8 @@ __device__ __forceinline__ float step_terms(const float (&pR)[V], const float (&
 template <int V>
 constexpr int loss_blocks() { return V >= 8 ? 2 : (V == 1 ? 8 : 4); }
 
-template <int V, bool ALL_VALID>
+// ST: the Spatio term too (heads = 3), fixed at compile time.
+template <int V, bool ALL_VALID, bool ST>
 __global__ void __launch_bounds__(32 * kLossWarps, loss_blocks<V>()) cache_loss_kernel(const LossArgs a) {
     const int lane = threadIdx.x & 31;
     const int task = blockIdx.x * kLossWarps + (threadIdx.x >> 5);
@@ -379,7 +380,7 @@ __global__ void __launch_bounds__(32 * kLossWarps, loss_blocks<V>()) cache_loss_
     const int t0 = c * a.chunk;
     const int t1 = min(T, t0 + a.chunk);
     const bool valid = ALL_VALID || lane < N / V;
-    const bool st = a.heads == 3;
+    constexpr bool st = ST;
     const bool want_grad = a.grad != nullptr;
     const float k2 = a.k2, cT = a.cT, cST = a.cST, gT = a.gT, gST = a.gST;
     const size_t row3 = (size_t)3 * N;
@@ -683,7 +684,7 @@ __device__ __forceinline__ float2 rows_step(const float (&pR)[kRowE], const RowS
     return make_float2(lT, lST);
 }
 
-template <int NL, int KP>
+template <int NL, int KP, bool ST>
 __global__ void __launch_bounds__(32 * kRowWarps, 3) cache_loss_rows_kernel(const LossArgs a) {
     constexpr int CPW = 32 / NL;                         // tasks per warp
     const int lane = threadIdx.x & 31;
@@ -699,7 +700,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 3) cache_loss_rows_kernel(cons
     const int b = active ? jl / L : 0, l = active ? jl % L : 0;
     const int t0 = c * a.chunk;
     const int t1 = min(T, t0 + a.chunk);
-    const bool st = a.heads == 3;
+    constexpr bool st = ST;
     const bool wr = active && a.grad != nullptr;
     const size_t row3 = (size_t)3 * N;
     const size_t tok = (size_t)L * row3;
@@ -849,13 +850,13 @@ __global__ void __launch_bounds__(32 * kRowWarps, 3) cache_loss_rows_kernel(cons
 // Token chunks of the short-row kernel: as many as give every resident warp
 // one (a single wave, each warp running one chunk of its 32 / NL chains),
 // chunks of at least 32 tokens so the halo step costs <= 1/32.
-template <int NL, int KP>
+template <int NL, int KP, bool ST>
 int launch_loss_rows(LossArgs& a, cudaStream_t stream) {
     constexpr int CPW = 32 / NL;
     static std::atomic<int> blocks_per_sm{0};
     if (blocks_per_sm.load() == 0) {
         int n = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, cache_loss_rows_kernel<NL, KP>,
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, cache_loss_rows_kernel<NL, KP, ST>,
                                                           32 * kRowWarps, 0) != cudaSuccess)
             return CRC_ECUDA;
         blocks_per_sm.store(n > 0 ? n : 1);
@@ -872,18 +873,24 @@ int launch_loss_rows(LossArgs& a, cudaStream_t stream) {
     const int grid = (int)((warps + kRowWarps - 1) / kRowWarps);
     {
         ProfScope prof(CRC_KERNEL_LOSS, stream);
-        cache_loss_rows_kernel<NL, KP><<<grid, 32 * kRowWarps, 0, stream>>>(a);
+        cache_loss_rows_kernel<NL, KP, ST><<<grid, 32 * kRowWarps, 0, stream>>>(a);
     }
     note_launch();
     return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
 }
 
+template <int NL, bool ST>
+int launch_loss_rows_st(LossArgs& a, cudaStream_t stream) {
+    if (a.top_b <= 2) return launch_loss_rows<NL, 2, ST>(a, stream);
+    if (a.top_b <= 4) return launch_loss_rows<NL, 4, ST>(a, stream);
+    if (a.top_b <= 8) return launch_loss_rows<NL, 8, ST>(a, stream);
+    return launch_loss_rows<NL, 16, ST>(a, stream);
+}
+
 template <int NL>
 int launch_loss_rows_kp(LossArgs& a, cudaStream_t stream) {
-    if (a.top_b <= 2) return launch_loss_rows<NL, 2>(a, stream);
-    if (a.top_b <= 4) return launch_loss_rows<NL, 4>(a, stream);
-    if (a.top_b <= 8) return launch_loss_rows<NL, 8>(a, stream);
-    return launch_loss_rows<NL, 16>(a, stream);
+    return a.heads == 3 ? launch_loss_rows_st<NL, true>(a, stream)
+                        : launch_loss_rows_st<NL, false>(a, stream);
 }
 
 // Means L_T, L_ST: fixed-order sums of the per-task sums (deterministic).
@@ -920,7 +927,10 @@ int launch_loss_t(const LossArgs& a, cudaStream_t stream) {
     const int grid = (tasks + kLossWarps - 1) / kLossWarps;
     {
         ProfScope prof(CRC_KERNEL_LOSS, stream);
-        cache_loss_kernel<V, ALL_VALID><<<grid, 32 * kLossWarps, 0, stream>>>(a);
+        if (a.heads == 3)
+            cache_loss_kernel<V, ALL_VALID, true><<<grid, 32 * kLossWarps, 0, stream>>>(a);
+        else
+            cache_loss_kernel<V, ALL_VALID, false><<<grid, 32 * kLossWarps, 0, stream>>>(a);
     }
     note_launch();
     return cudaGetLastError() == cudaSuccess ? CRC_OK : CRC_ECUDA;
